@@ -1,0 +1,140 @@
+"""Pins of the oracle's GA operators (Sec. IV-C: tournament selection,
+crossover, mutation, elitism) by properties that any correct implementation of
+the stated operators must have.  The whole-GA trajectory is not pinned beyond
+these operator properties (a fitness difference of one ulp can flip a
+tournament)."""
+import math
+
+import numpy as np
+import pytest
+
+from paper_2609_02109_gb300 import workload as W
+
+
+def _ga(**kw):
+    g = dict(W.GA_PARAMS)
+    g.update(kw)
+    return g
+
+
+@pytest.fixture(scope="module")
+def prob():
+    return W.paper_scale()
+
+
+def test_rng_counter_fields_are_distinct(oracle_mod):
+    seen = set()
+    for gen in (0, 1, 99):
+        for slot in (0, 1, 1023, 2 ** 20 - 1):
+            for purpose in range(6):
+                for j in (0, 1, 255):
+                    seen.add(oracle_mod.rng(5, gen, slot, purpose, j))
+    assert len(seen) == 3 * 4 * 6 * 3
+
+
+def test_init_is_uniform_over_each_option_range(oracle_mod, prob):
+    o = oracle_mod.Oracle(prob)
+    pop = o.ga_init(_ga(pop=20000), seed=3)
+    ks = prob["n_options"]
+    assert pop.shape == (20000, 5)
+    for i, k in enumerate(ks):
+        assert pop[:, i].min() == 0 and pop[:, i].max() == k - 1
+        counts = np.bincount(pop[:, i], minlength=k)
+        exp = 20000 / k
+        chi2 = float(((counts - exp) ** 2 / exp).sum())
+        assert chi2 < k + 8 * math.sqrt(2 * k)  # loose chi-square bound
+
+
+def test_elitism_keeps_the_fittest_lowest_slot(oracle_mod, prob):
+    o = oracle_mod.Oracle(prob)
+    g = _ga(pop=64)
+    pop = o.ga_init(g, seed=1)
+    fit = np.linspace(-1, 1, 64)
+    fit[[17, 40]] = 5.0  # tie: slot 17 must win
+    nxt = o.ga_step(g, 1, 0, pop, fit)
+    assert list(nxt[0]) == list(pop[17])
+    g0 = _ga(pop=64, elitism=0)
+    nxt0 = o.ga_step(g0, 1, 0, pop, fit)
+    assert np.array_equal(nxt0[1:], nxt[1:])  # children do not depend on elitism
+
+
+def test_children_come_from_two_parents_without_mutation(oracle_mod):
+    """With p_m = 0 every child gene is copied from one of two parents.  Slot s
+    carries genome (s, s, ..., s), so each child names at most two slots."""
+    p = W.make_problem([256] * 6, 8, 16, 0, 5, 1e9)
+    o = oracle_mod.Oracle(p)
+    g = _ga(pop=256, mutation_p=0.0)
+    pop = np.repeat(np.arange(256, dtype=np.int32)[:, None], 6, axis=1)
+    fit = np.arange(256, dtype=np.float64)
+    nxt = o.ga_step(g, 9, 3, pop, fit)
+    mixed = 0
+    for c in range(1, 256):
+        src = set(nxt[c].tolist())
+        assert len(src) <= 2
+        mixed += len(src) == 2
+    # uniform crossover of two distinct parents gives a mix with prob 1 - 2 / 2**6
+    assert mixed > 0.8 * 255
+    # tournament of 4 over fitness = slot: the winner is the max of 4 uniform
+    # draws, mean about 4/5 of the range
+    parents = np.array([v for c in range(1, 256) for v in set(nxt[c].tolist())])
+    assert 0.74 * 255 < parents.mean() < 0.86 * 255
+
+
+def test_tournament_of_one_is_uniform(oracle_mod):
+    p = W.make_problem([256], 8, 16, 0, 5, 1e9)
+    o = oracle_mod.Oracle(p)
+    g = _ga(pop=256, tournament=1, mutation_p=0.0)
+    pop = np.arange(256, dtype=np.int32)[:, None]
+    nxt = o.ga_step(g, 2, 0, pop, np.arange(256, dtype=np.float64))
+    assert 0.4 * 255 < nxt[1:, 0].mean() < 0.6 * 255
+
+
+def test_mutation_rate(oracle_mod, prob):
+    """Identical parents: a gene differs from the parent exactly when it mutated to
+    another value, with probability p_m * (1 - 1/K_i)."""
+    o = oracle_mod.Oracle(prob)
+    P = 8192
+    g = _ga(pop=P, mutation_p=0.05)
+    pop = np.tile(np.array([3, 4, 5, 6, 7], dtype=np.int32), (P, 1))
+    nxt = o.ga_step(g, 11, 7, pop, np.zeros(P))
+    ks = prob["n_options"]
+    for i, k in enumerate(ks):
+        rate = float((nxt[1:, i] != pop[0, i]).mean())
+        exp = 0.05 * (1 - 1 / k)
+        sd = math.sqrt(exp * (1 - exp) / (P - 1))
+        assert abs(rate - exp) < 5 * sd
+        assert nxt[:, i].min() >= 0 and nxt[:, i].max() < k
+
+
+def test_full_mutation_is_uniform(oracle_mod, prob):
+    o = oracle_mod.Oracle(prob)
+    P = 12000
+    g = _ga(pop=P, mutation_p=1.0, elitism=0)
+    pop = np.zeros((P, 5), dtype=np.int32)
+    nxt = o.ga_step(g, 4, 0, pop, np.zeros(P))
+    k = int(prob["n_options"][0])
+    counts = np.bincount(nxt[:, 0], minlength=k)
+    exp = P / k
+    assert float(((counts - exp) ** 2 / exp).sum()) < k + 8 * math.sqrt(2 * k)
+
+
+def test_ga_step_is_deterministic_and_seeded(oracle_mod, prob):
+    o = oracle_mod.Oracle(prob)
+    g = _ga(pop=128)
+    pop = o.ga_init(g, 5)
+    fit = np.random.default_rng(0).standard_normal(128)
+    a = o.ga_step(g, 5, 2, pop, fit)
+    assert np.array_equal(a, o.ga_step(g, 5, 2, pop, fit))
+    assert not np.array_equal(a, o.ga_step(g, 6, 2, pop, fit))
+    assert not np.array_equal(a, o.ga_step(g, 5, 3, pop, fit))
+
+
+def test_ga_finds_optimum_of_tiny_space(oracle_mod):
+    """216 candidates, population 64 over 30 generations: the GA must reach the
+    exhaustive optimum (the argmax over the same landscape, Sec. IV-C)."""
+    p = W.tiny()
+    o = oracle_mod.Oracle(p)
+    ti, ts, _ = o.exhaustive(1)
+    J, genome = o.ga_run(_ga(pop=64, gens=30), seed=1000)
+    assert J == ts[0]
+    assert list(genome) == list(o.decode(int(ti[0])))
