@@ -1,0 +1,200 @@
+/*
+ * mf.h -- C ABI of the GB300 MeanField joint-configuration scorer.
+ *
+ * The library scores joint co-location configurations of N models that share
+ * one GPU, following arXiv 2609.02109:
+ *   - the joint space Lambda = prod_i Lambda_i of per-model option sets (Sec. II, Eq. 1),
+ *     enumerated as a mixed-radix index, last model fastest;
+ *   - the aggregate GPU state of a candidate (summed SM share, VRAM and bandwidth
+ *     demand of the chosen options, plus N) (Eq. 2, in the coupled reading where the
+ *     aggregate is formed from the candidate's own demands);
+ *   - one MeanField predictor per model, (thr_i, lat_i) = g_i(local_i, aggregate)
+ *     (Sec. III-B, Eq. 6): an MLP Linear-ReLU-[Linear-ReLU]-Linear with an optional
+ *     sigmoid on the two outputs;
+ *   - the hard constraints sum_i VRAM_i <= R and lat_i <= SLA_i (Eq. 4), infeasible
+ *     candidates scoring -inf (Sec. II);
+ *   - the objective J = sum_i w_i thr_i (the throughput-weighted term of Eq. 3), or,
+ *     with MF_OBJ_SOFT_LAT, J = sum_i w_i thr_i - lambda sum_i max(0, lat_i - SLA_i)
+ *     with only the VRAM constraint hard;
+ *   - exhaustive argmax / top-k / feasible count over Lambda (Sec. II, Sec. IV-C), and
+ *     the GA scheduler's per-generation fitness batch and operators (Sec. IV-C).
+ *
+ * Conventions for every call:
+ *   - Functions return an mf_status and never abort or throw.  mf_last_error()
+ *     returns a human-readable detail string for the calling thread's last failure.
+ *   - "d_" pointers are device pointers owned by the caller; they must stay valid
+ *     until the work on `stream` completes.  `stream` is a cudaStream_t (NULL =
+ *     the legacy default stream).  Host pointers are caller-owned too.
+ *   - A context is thread-compatible: calls on one context must not run
+ *     concurrently from several host threads.  Different contexts are independent.
+ *   - Indices are uint64; digits/genes are int32 with 0 <= o_i < K_i.
+ *   - The total order of results is (J descending, index ascending).  Infeasible
+ *     candidates have J = -INFINITY and never enter a top-k.  Unfilled top-k slots
+ *     are (UINT64_MAX, -INFINITY).  No feasible candidate is not an error.
+ *   - A candidate whose J is NaN counts as infeasible.
+ */
+#ifndef MF_H
+#define MF_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  MF_OK = 0,
+  MF_EINVAL = 1,        /* invalid argument (see each call) */
+  MF_ENOMEM = 2,        /* device or host allocation failed */
+  MF_ECUDA = 3,         /* a CUDA runtime call failed; see mf_last_error() */
+  MF_EUNSUPPORTED = 4,  /* valid but unsupported shape/precision combination */
+  MF_ETIMEOUT = 5,      /* a bounded device-side wait gave up */
+  MF_EDEVICE = 6        /* the device reported an invalid input (e.g. an index >= |Lambda|) */
+} mf_status;
+
+typedef enum { MF_FP32 = 0, MF_BF16 = 1 } mf_precision;
+typedef enum { MF_OBJ_WEIGHTED_THR = 0, MF_OBJ_SOFT_LAT = 1 } mf_objective;
+typedef enum { MF_ACT_IDENTITY = 0, MF_ACT_SIGMOID = 1 } mf_out_act;
+
+#define MF_MAX_MODELS 16
+#define MF_MAX_OPTIONS 255
+#define MF_MAX_D_LOCAL 28
+#define MF_MAX_HIDDEN 256
+#define MF_MAX_TOPK 1024
+
+typedef struct mf_ctx mf_ctx;
+
+/* Problem description (Sec. II and Sec. III-B).  All arrays are host memory and
+ * are deep-copied by mf_create; the caller may free them afterwards. */
+typedef struct {
+  int32_t n_models;            /* N, 1..MF_MAX_MODELS */
+  const int32_t *n_options;    /* [N] K_i = |Lambda_i|, each 1..MF_MAX_OPTIONS */
+  int32_t d_local;             /* d_L, 1..MF_MAX_D_LOCAL; predictor input d_in = d_L + 4 */
+  int32_t hidden1;             /* first hidden width, 1..MF_MAX_HIDDEN */
+  int32_t hidden2;             /* second hidden width, 0 (one hidden layer) or 1..MF_MAX_HIDDEN */
+  const float *local_feats;    /* [sum K_i][d_L] row-major, model-major option rows */
+  const float *demand;         /* [sum K_i][3]: SM share, VRAM GB, bandwidth GB/s */
+  const float *weights;        /* per model, PyTorch Linear layout (weight[out][in]):
+                                  W1[h1][d_in], b1[h1], (W2[h2][h1], b2[h2]), W3[2][h], b3[2];
+                                  output 0 = throughput, output 1 = latency */
+  const float *agg_scale;      /* [4] multipliers of (sum SM, sum VRAM, sum BW, N) before the
+                                  predictor; NULL = (1/(0.6N), 1/(20N), 1/(1500N), 1/8) */
+  const float *sla;            /* [N] latency ceilings SLA_i */
+  const float *obj_w;          /* [N] objective weights w_i */
+  float vram_cap;              /* R, GB; feasibility needs sum VRAM <= R */
+  float soft_penalty;          /* lambda of MF_OBJ_SOFT_LAT (ignored otherwise) */
+  int32_t out_act;             /* mf_out_act */
+  int32_t objective;           /* mf_objective */
+  int32_t precision;           /* mf_precision of the scoring kernels */
+  int32_t device;              /* CUDA device ordinal, or -1 for the current device */
+} mf_problem;
+
+/* Result of an exhaustive search.  topk_idx/topk_score are caller-owned host
+ * arrays of k entries (either may be NULL). */
+typedef struct {
+  uint64_t best_idx;           /* UINT64_MAX if no feasible candidate */
+  float best_score;            /* -INFINITY if no feasible candidate */
+  uint64_t feasible_count;
+  int32_t k;
+  uint64_t *topk_idx;
+  float *topk_score;
+} mf_result;
+
+/* GA parameters (Sec. IV-C): population, generations, tournament size, per-gene
+ * mutation probability, elitism (0 or 1).  Crossover is uniform. */
+typedef struct {
+  int32_t pop;                 /* 2..65536 */
+  int32_t gens;                /* >= 1 fitness evaluations */
+  int32_t tournament;          /* 1..256 */
+  double mutation_p;           /* [0, 1] */
+  int32_t elitism;             /* 0 or 1 */
+} mf_ga_params;
+
+/* Name of a status code (static string). */
+const char *mf_status_string(mf_status s);
+
+/* Detail of the calling thread's last failing call ("" if none). */
+const char *mf_last_error(void);
+
+/* Validate `p` (Sec. II problem statement), copy it to the device and prepare
+ * the kernels.  MF_EINVAL: N, K_i, d_L or widths out of range, NULL arrays, or
+ * prod K_i overflowing uint64.  MF_EUNSUPPORTED: MF_BF16 with a shape the
+ * tensor-core kernel does not cover.  On success *out owns device memory until
+ * mf_destroy. */
+mf_status mf_create(const mf_problem *p, mf_ctx **out);
+
+/* Release the context and its device memory (synchronises the device first).
+ * NULL is accepted. */
+mf_status mf_destroy(mf_ctx *ctx);
+
+/* |Lambda| = prod_i K_i (Eq. 1). */
+mf_status mf_space_size(const mf_ctx *ctx, uint64_t *out);
+
+/* Replace SLA_i and w_i (a new scheduling scenario); NULL keeps the old array.
+ * Takes effect for calls issued afterwards. */
+mf_status mf_set_objective(mf_ctx *ctx, const float *sla, const float *obj_w);
+
+/* Score n candidates given by index (Eqs. 1-6 and the constraints of Eq. 4).
+ *   d_idx      [n] uint64 indices into Lambda
+ *   d_score    [n] J (or -INFINITY when infeasible)
+ *   d_feasible [n] 1 feasible / 0 not (may be NULL)
+ *   d_pred     [n][N][2] (thr_i, lat_i) per model (may be NULL)
+ * Asynchronous on `stream`.  An index >= |Lambda| scores -INFINITY, infeasible,
+ * and raises the context's device status, read by mf_check_device_status. */
+mf_status mf_score_batch(mf_ctx *ctx, const uint64_t *d_idx, uint64_t n, float *d_score,
+                         uint8_t *d_feasible, float *d_pred, void *stream);
+
+/* Exhaustive surrogate search over [lo, hi) of Lambda (the argmax of Sec. II,
+ * extended to top-k and the feasible count), processed in launches of `chunk`
+ * candidates (0 = the library's default) while the running top-k and count are
+ * carried across launches.  k in 1..MF_MAX_TOPK.  Synchronous: returns after
+ * `out` is filled.  The BF16 precision keeps a shortlist of max(8k, 256)
+ * candidates by tensor-core score and re-scores it in fp32, so reported scores
+ * and the top-k order are the fp32 ones; its feasible count is taken at bf16
+ * precision. */
+mf_status mf_search_range(mf_ctx *ctx, uint64_t lo, uint64_t hi, int32_t k, uint64_t chunk,
+                          mf_result *out, void *stream);
+
+/* mf_search_range over the whole space [0, |Lambda|). */
+mf_status mf_search_exhaustive(mf_ctx *ctx, int32_t k, uint64_t chunk, mf_result *out,
+                               void *stream);
+
+/* GA fitness batch (Sec. IV-C): d_pop [P][N] int32 genes -> d_fitness [P] (J or
+ * -INFINITY).  Asynchronous.  A gene outside [0, K_i) gives -INFINITY and raises
+ * the device status. */
+mf_status mf_ga_generation(mf_ctx *ctx, const int32_t *d_pop, int32_t P, float *d_fitness,
+                           void *stream);
+
+/* Initial population: gene i of slot c is uniform on [0, K_i) from the
+ * counter-based generator (seed, generation 0, c, purpose 0, i).  Asynchronous. */
+mf_status mf_ga_init(mf_ctx *ctx, const mf_ga_params *g, uint64_t seed, int32_t *d_pop,
+                     void *stream);
+
+/* One GA generation (Sec. IV-C operators): from population `gen` and its
+ * fitness to population gen + 1.  Slot 0 keeps the fittest individual (lowest
+ * slot among equals) when elitism is on; every other slot draws two parents by
+ * tournament (draws with replacement, best fitness, lowest slot among equals),
+ * takes each gene from either parent with probability 1/2, and redraws a gene
+ * uniformly with probability mutation_p.  All draws are SplitMix64 outputs at
+ * counter (gen + 1) << 32 | slot << 12 | purpose << 8 | j of the stream `seed`.
+ * Asynchronous.  d_next must not alias d_pop. */
+mf_status mf_ga_step(mf_ctx *ctx, const mf_ga_params *g, uint64_t seed, int32_t gen,
+                     const int32_t *d_pop, const float *d_fitness, int32_t *d_next,
+                     void *stream);
+
+/* A complete GA decision: init, then g->gens fitness batches with a generation
+ * step between consecutive ones; returns the fittest individual of the last
+ * population (lowest slot among equals) in best_genome[N] (host) and its
+ * fitness.  Synchronous. */
+mf_status mf_ga_run(mf_ctx *ctx, const mf_ga_params *g, uint64_t seed, int32_t *best_genome,
+                    float *best_fitness, void *stream);
+
+/* Synchronise `stream`, then return MF_EDEVICE if any asynchronous call since the
+ * last check saw an invalid index or gene (and clear that flag), else MF_OK. */
+mf_status mf_check_device_status(mf_ctx *ctx, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* MF_H */

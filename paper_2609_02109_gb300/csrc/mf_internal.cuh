@@ -1,0 +1,260 @@
+// Internal declarations of the CUDA path (not part of the public ABI).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <string>
+#include <vector>
+
+#include "../../include/mf.h"
+
+namespace mf {
+
+constexpr uint64_t kEmptyIdx = ~0ull;
+constexpr int kScoreThreads = 512;   // CTA size of the CUDA-core scorer
+constexpr int kWideWarps = 8;        // warps per CTA of the warp-per-(candidate, model) scorer
+
+// Everything a kernel needs about a problem, passed by value (a few hundred bytes).
+struct Params {
+  int32_t n_models, d_local, h1, h2, d_in;
+  int32_t objective, out_act;
+  float vram_cap, soft_penalty;
+  float agg_scale[4];
+  int32_t K[MF_MAX_MODELS];           // options per model
+  int32_t off[MF_MAX_MODELS];         // first option row of each model
+  uint64_t stride[MF_MAX_MODELS];     // prod_{j>i} K_j (mixed-radix place values)
+  float sla[MF_MAX_MODELS];
+  float w[MF_MAX_MODELS];
+  uint64_t total;                     // |Lambda|
+  int64_t per_model;                  // floats per packed predictor
+  const float* x;                     // [sumK][d_local]
+  const float4* dem;                  // [sumK] (sm, vram, bw, 0)
+  const float* w32;                   // predictors, packed as given
+  const float* wT;                    // predictors with W1, W2 transposed ([in][out])
+  uint32_t* status;                   // device status word (bit 0: bad index/gene)
+};
+
+// Device status bits.
+constexpr uint32_t kStatusBadInput = 1u;
+constexpr uint32_t kStatusTimeout = 2u;
+
+// ---------------------------------------------------------------------------
+// Device helpers
+// ---------------------------------------------------------------------------
+
+// (J, idx) total order: J descending, then index ascending.
+__device__ __forceinline__ bool precedes(float ja, uint64_t ia, float jb, uint64_t ib) {
+  return ja > jb || (ja == jb && ia < ib);
+}
+
+// ReLU that keeps NaN (so a NaN weight reaches the outputs and marks the
+// candidate infeasible).
+__device__ __forceinline__ float relu(float v) { return v < 0.f ? 0.f : v; }
+
+// Digit of model i of index idx (C order: last model fastest).
+__device__ __forceinline__ int digit_of(const Params& P, uint64_t idx, int i) {
+  if (P.total <= 0x100000000ull) {
+    uint32_t q = (uint32_t)idx / (uint32_t)P.stride[i];
+    return (int)(q % (uint32_t)P.K[i]);
+  }
+  return (int)((idx / P.stride[i]) % (uint64_t)P.K[i]);
+}
+
+// Output unit of the predictor: identity or sigmoid (the paper's output layer).
+__device__ __forceinline__ float out_act(const Params& P, float v) {
+  return P.out_act == MF_ACT_SIGMOID ? 1.f / (1.f + expf(-v)) : v;
+}
+
+// Objective and constraints of one candidate from per-model outputs.
+struct Acc {
+  float J, pen;
+  bool sla_ok;
+  __device__ __forceinline__ void init() { J = 0.f; pen = 0.f; sla_ok = true; }
+  // thr, lat: predictor outputs after the output activation.
+  __device__ __forceinline__ void add(const Params& P, int i, float thr, float lat) {
+    J = fmaf(P.w[i], thr, J);
+    sla_ok = sla_ok && (lat <= P.sla[i]);
+    float over = lat - P.sla[i];
+    pen += over > 0.f ? over : 0.f;
+  }
+  // Returns feasibility; J becomes the final score (-inf when infeasible).
+  __device__ __forceinline__ bool finish(const Params& P, float vram_sum) {
+    bool feas = vram_sum <= P.vram_cap;
+    if (P.objective == MF_OBJ_WEIGHTED_THR) feas = feas && sla_ok;
+    else J = fmaf(-P.soft_penalty, pen, J);
+    if (J != J) feas = false;
+    if (!feas) J = -INFINITY;
+    return feas;
+  }
+};
+
+// SplitMix64 output number ctr of the sequence whose state starts at seed
+// (Steele, Lea and Flood, OOPSLA 2014).
+__device__ __forceinline__ uint64_t splitmix64(uint64_t seed, uint64_t ctr) {
+  uint64_t z = seed + (ctr + 1ull) * 0x9E3779B97F4A7C15ull;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+__device__ __forceinline__ uint64_t ga_rng(uint64_t seed, uint32_t gen, uint32_t slot,
+                                           uint32_t purpose, uint32_t j) {
+  uint64_t ctr = ((uint64_t)gen << 32) | ((uint64_t)(slot & 0xFFFFFu) << 12) |
+                 ((uint64_t)(purpose & 0xFu) << 8) | (uint64_t)(j & 0xFFu);
+  return splitmix64(seed, ctr);
+}
+
+__device__ __forceinline__ int ga_unif(uint64_t r, uint32_t k) {
+  return (int)(((r >> 32) * (uint64_t)k) >> 32);
+}
+
+enum { kGaInit = 0, kGaTourA = 1, kGaTourB = 2, kGaCross = 3, kGaMut = 4, kGaMutVal = 5 };
+
+// ---------------------------------------------------------------------------
+// Per-CTA running top-k in shared memory (sorted by the total order), fed by
+// a queue of candidates that beat the current k-th entry.
+// ---------------------------------------------------------------------------
+struct CtaTopK {
+  float* ls; uint64_t* li;   // current list [k]
+  float* ns; uint64_t* ni;   // merge output [k]
+  float* qs; uint64_t* qi;   // queue [qcap]
+  int* qn;
+  int k;
+};
+
+// Merge the queue into the list.  Called by `nthr` threads (ids 0..nthr-1) after a
+// barrier that made the queue visible; `sync()` is a barrier over those threads.
+template <class Sync>
+__device__ void topk_merge(const CtaTopK& t, int tid, int nthr, Sync sync) {
+  const int k = t.k;
+  const int q = *t.qn;
+  for (int e = tid; e < k; e += nthr) { t.ns[e] = -INFINITY; t.ni[e] = kEmptyIdx; }
+  sync();
+  for (int e = tid; e < k + q; e += nthr) {
+    float s; uint64_t id; int rank;
+    if (e < k) {
+      s = t.ls[e]; id = t.li[e];
+      if (id == kEmptyIdx) continue;
+      rank = e;
+    } else {
+      s = t.qs[e - k]; id = t.qi[e - k];
+      int lo = 0, hi = k;
+      while (lo < hi) {
+        int mid = (lo + hi) >> 1;
+        if (precedes(t.ls[mid], t.li[mid], s, id)) lo = mid + 1; else hi = mid;
+      }
+      rank = lo;
+    }
+    for (int j = 0; j < q && rank < k; ++j) rank += precedes(t.qs[j], t.qi[j], s, id) ? 1 : 0;
+    if (rank < k) { t.ns[rank] = s; t.ni[rank] = id; }
+  }
+  sync();
+  for (int e = tid; e < k; e += nthr) { t.ls[e] = t.ns[e]; t.li[e] = t.ni[e]; }
+  if (tid == 0) *t.qn = 0;
+  sync();
+}
+
+}  // namespace mf
+
+// ---------------------------------------------------------------------------
+// Host side
+// ---------------------------------------------------------------------------
+struct mf_ctx {
+  int device = 0;
+  int num_sms = 0;
+  mf::Params P{};                 // device pointers filled in
+  int32_t precision = MF_FP32;
+  std::vector<int32_t> K;
+  int sumK = 0;
+  // device buffers owned by the context
+  float* d_x = nullptr;
+  float4* d_dem = nullptr;
+  float* d_w32 = nullptr;
+  float* d_wT = nullptr;
+  uint32_t* d_status = nullptr;
+  void* d_tc = nullptr;           // packed bf16 operand images (tensor-core path)
+  size_t tc_bytes = 0;
+  // growable scratch (search lists, merge buffers, shortlist)
+  void* d_scratch = nullptr;
+  size_t scratch_bytes = 0;
+  // pinned host staging for results
+  void* h_stage = nullptr;
+  size_t h_stage_bytes = 0;
+  // GA: populations, fitness, per-model outputs, result, and the captured graph
+  int32_t* d_pop[2] = {nullptr, nullptr};
+  float* d_fit = nullptr;
+  float* d_pred = nullptr;
+  void* d_ga_out = nullptr;       // best genome [N] int32, then its fitness (float), then the seed (u64)
+  int ga_cap = 0;
+  cudaStream_t cap_stream = nullptr;
+  cudaGraphExec_t ga_exec = nullptr;
+  uint64_t params_version = 0;
+  uint64_t ga_version = ~0ull;
+  mf_ga_params ga_key{};
+};
+
+namespace mf {
+
+// Thread-local detail string of the last failure.
+void set_error(const std::string& msg);
+mf_status cuda_fail(cudaError_t e, const char* what);
+
+#define MF_CUDA(call)                                         \
+  do {                                                        \
+    cudaError_t _e = (call);                                  \
+    if (_e != cudaSuccess) return ::mf::cuda_fail(_e, #call); \
+  } while (0)
+
+// Scratch management.
+mf_status ensure_scratch(mf_ctx* c, size_t bytes);
+mf_status ensure_host_stage(mf_ctx* c, size_t bytes);
+
+// CUDA-core scorer (exact fp32 path).
+struct RangeArgs {
+  uint64_t base, len;
+  int k;
+  int first;            // 1: initialise the per-CTA lists
+  float* lists_s;       // [grid][k]
+  uint64_t* lists_i;    // [grid][k]
+  unsigned long long* count;
+};
+bool f32_supported(const Params& P);
+size_t f32_smem_bytes(const Params& P, int k, bool& resident);
+int f32_grid(const mf_ctx* c);
+mf_status f32_prepare(mf_ctx* c);
+mf_status f32_search_chunk(mf_ctx* c, const RangeArgs& a, cudaStream_t s);
+mf_status f32_score_list(mf_ctx* c, const uint64_t* idx, const int32_t* genes, uint64_t n,
+                         float* score, uint8_t* feas, float* pred, cudaStream_t s);
+// Exact re-scoring of a shortlist that may contain empty slots (index UINT64_MAX),
+// which score -inf without raising the device status.  pred: scratch [n][N][2].
+mf_status f32_score_list_ex(mf_ctx* c, const uint64_t* idx, uint64_t n, float* score, float* pred,
+                            cudaStream_t s);
+
+// Merge of per-CTA sorted lists into one sorted top-k.
+mf_status merge_lists(mf_ctx* c, const float* ls, const uint64_t* li, int nlists, int k,
+                      float* tmp_s, uint64_t* tmp_i, float* out_s, uint64_t* out_i,
+                      cudaStream_t s);
+// Sort n (score, idx) pairs by the total order and keep the first k (n <= 8192).
+mf_status select_topk(mf_ctx* c, const float* in_s, const uint64_t* in_i, int n, int k,
+                      float* out_s, uint64_t* out_i, cudaStream_t s);
+
+// Tensor-core scorer (bf16 path).
+bool tc_supported(const Params& P, std::string* why);
+mf_status tc_prepare(mf_ctx* c);
+int tc_grid(const mf_ctx* c);
+mf_status tc_search_chunk(mf_ctx* c, const RangeArgs& a, cudaStream_t s);
+mf_status tc_score_list(mf_ctx* c, const uint64_t* idx, uint64_t n, float* score,
+                        uint8_t* feas, float* pred, cudaStream_t s);
+
+// GA kernels.
+mf_status ga_init(mf_ctx* c, const mf_ga_params* g, uint64_t seed, int32_t* pop, cudaStream_t s);
+mf_status ga_step(mf_ctx* c, const mf_ga_params* g, uint64_t seed, int32_t gen,
+                  const int32_t* pop, const float* fit, int32_t* next, cudaStream_t s);
+mf_status ga_best(mf_ctx* c, const int32_t* pop, const float* fit, int P, int32_t* out_genome,
+                  float* out_fit, cudaStream_t s);
+// Whole GA decision as one CUDA graph launch on `s`; the result lands in c->d_ga_out
+// and the pinned staging buffer is sized for it.
+mf_status ga_run_graph(mf_ctx* c, const mf_ga_params* g, uint64_t seed, cudaStream_t s);
+
+}  // namespace mf
