@@ -1,0 +1,348 @@
+"""Benchmark of the MeanField joint-configuration scorer on GB300.
+
+One step = one exhaustive surrogate search over the large workload: N = 6
+models with 24 options each (24**6 = 191,102,976 joint configurations),
+12->64->64->2 predictors, VRAM cap 180 GB, top-32 and the feasible count,
+enumerated in launches of 2**24 candidates.  All inputs are seeded synthetic
+draws (paper_2609_02109_gb300.workload).  The GA decision latency (N = 5,
+population 1024, 100 generations, 8 scenarios) is measured after the timed
+steps and reported in the same JSON line.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--precision bf16|fp32]
+    python bench.py --impl reference ...   # the CPU oracle as the reference arm
+
+Multi-GPU (torchrun, one rank per GPU): every rank searches its own scenario
+(independent problems, no collective in the data path): weak scaling.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2609_02109_gb300 import workload as W  # noqa: E402
+
+METRIC = "joint configs scored/s (N=6 exhaustive, % of roofline); p50 GA decision ms"
+UNIT = "configs/s"
+K_TOP = 32
+CHUNK = 1 << 24
+L2_FLUSH_BYTES = 256 << 20
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f), "measured"
+    except OSError:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+                "sm_max_mhz": 2070.0}, "fallback"
+
+
+def flops_per_candidate(prob) -> int:
+    """Algorithmic FLOPs of one candidate: 2 x (multiply-adds of every layer) x N."""
+    din = prob["d_local"] + 4
+    h1, h2 = prob["hidden1"], prob["hidden2"]
+    macs = din * h1 + (h1 * h2 + h2 * 2 if h2 else h1 * 2)
+    return 2 * macs * int(prob["n_options"].size)
+
+
+def workload_config(prec):
+    return {
+        "workload": "large exhaustive: N=6 models x 24 options (24^6 = 191,102,976 joint configs), "
+                    "per-model MLP 12->64->64->2, VRAM cap 180 GB, SLA~U(0.5,2), w~U(0.5,1.5), "
+                    "top-32 + feasible count, launches of 2^24 candidates",
+        "precision": prec,
+        "seed": 3,
+        "l2": "flushed between timed steps (256 MiB device write); scoring inputs are on-chip "
+              "tables and weights",
+    }
+
+
+# ---------------------------------------------------------------------------
+# Clock sampling during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.out = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}", "--format=csv,noheader",
+                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except OSError:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.out.append(line.strip())
+
+    def __exit__(self, *exc):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.out:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1].split()[0]))
+                mx.append(float(parts[2].split()[0]))
+            except ValueError:
+                continue
+            for name, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# CPU baseline: the oracle on a bounded sample of the same workload
+# ---------------------------------------------------------------------------
+def cpu_baseline(prob, target_s=12.0):
+    from oracle.oracle import Oracle
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    o = Oracle(prob, nthreads=cores)
+    t = time.perf_counter()
+    o.exhaustive(K_TOP, lo=0, hi=20000)
+    rate = 20000 / max(time.perf_counter() - t, 1e-6)
+    n = int(min(max(rate * target_s, 1e5), 5e7))
+    t = time.perf_counter()
+    o.exhaustive(K_TOP, lo=0, hi=n)
+    dt = time.perf_counter() - t
+    return {"value": n / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"fp64 C oracle exhaustive search (top-32 + count) over indices [0, {n}) "
+                      f"of the same N=6 space, {dt:.1f} s"}
+
+
+def run_reference(args):
+    """Reference arm: the CPU oracle, timed on the host cores, per step a bounded sample."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    from oracle.oracle import Oracle, build
+    build()
+    prob = W.large(precision="fp32")
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    o = Oracle(prob, nthreads=cores)
+    t = time.perf_counter()
+    o.exhaustive(K_TOP, lo=0, hi=20000)
+    rate = 20000 / max(time.perf_counter() - t, 1e-6)
+    budget = 150.0 / max(args.steps + args.warmup, 1)
+    n = int(min(max(rate * min(budget, 20.0), 5e4), 5e7))
+    for _ in range(args.warmup):
+        o.exhaustive(K_TOP, lo=0, hi=min(n, 20000))
+    times = []
+    for s in range(args.steps):
+        lo = (s * n) % (prob_size := 24 ** 6)
+        hi = min(lo + n, prob_size)
+        t = time.perf_counter()
+        o.exhaustive(K_TOP, lo=lo, hi=hi)
+        times.append(time.perf_counter() - t)
+    total = sum(times)
+    value = n * args.steps / total
+    sample = f"fp64 C oracle exhaustive search over {n} consecutive indices per step of the N=6 space"
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": workload_config("f64"),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+def ga_latency(mf, torch, device, decisions_per_scenario):
+    """p50/p99 of complete GA decisions (host call -> result on host) over 8 scenarios."""
+    g = W.GA_PARAMS
+    wall, dev = [], []
+    gaps = []
+    for sc in W.GA_SCENARIO_SEEDS:
+        prob = W.ga_scenario(sc)
+        with mf.Context(prob, device=device) as ctx:
+            best = ctx.search(1)["best_score"]
+            ctx.ga_run(g, 999)  # builds the graph
+            stream = torch.cuda.current_stream(device)
+            for j in range(decisions_per_scenario):
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                torch.cuda.synchronize(device)
+                t0 = time.perf_counter()
+                e0.record(stream)
+                J, genome = ctx.ga_run(g, W.GA_RUN_SEEDS[j % len(W.GA_RUN_SEEDS)])
+                e1.record(stream)
+                t1 = time.perf_counter()
+                e1.synchronize()
+                wall.append(1e3 * (t1 - t0))
+                dev.append(e0.elapsed_time(e1))
+                gaps.append(100.0 * (best - J) / abs(best) if best != 0 else 0.0)
+    q = lambda a, p: float(np.percentile(np.asarray(a), p))  # noqa: E731
+    return {"p50_ms": q(wall, 50), "p99_ms": q(wall, 99), "device_p50_ms": q(dev, 50),
+            "decisions": len(wall), "scenarios": len(W.GA_SCENARIO_SEEDS),
+            "gap_pct_avg": float(np.mean(gaps)), "gap_pct_worst": float(np.max(gaps)),
+            "config": "N=5 paper-scale problem (78,732 configs), pop 1024, 100 generations, "
+                      "tournament 4, uniform crossover, mutation 0.05, elitism 1, fp32 fitness",
+            "gap_vs": "exhaustive optimum of the same scenario (fp32)"}
+
+
+def run_gpu(args):
+    import torch
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    import __graft_entry__
+    if rank == 0 or world == 1:
+        __graft_entry__.build()
+    if dist:
+        dist.barrier()
+    from paper_2609_02109_gb300 import mf
+
+    prec = args.precision
+    prob = W.large(precision=prec)
+    if rank:
+        W.set_scenario(prob, 3 + 1000 * rank)
+    n_cand = 24 ** 6
+    device = local
+    stream = torch.cuda.current_stream(device)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=f"cuda:{device}")
+    with mf.Context(prob, device=device) as ctx:
+        for _ in range(args.warmup):
+            ctx.search(K_TOP, chunk=CHUNK)
+        step_ms, score_ms, launches, score_launches = [], [], 0, 0
+        res = None
+        with ClockSampler(device) as clk:
+            if dist:
+                dist.barrier()
+            torch.cuda.synchronize(device)
+            for _ in range(args.steps):
+                flush.fill_(1.0)  # L2 flush outside the timed events
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                res = ctx.search(K_TOP, chunk=CHUNK)
+                e1.record(stream)
+                e1.synchronize()
+                step_ms.append(e0.elapsed_time(e1))
+                st = ctx.stats()
+                score_ms.append(st["score_ms_last"])
+                launches += st["kernel_launches_last"]
+                score_launches += st["score_launches_last"]
+            torch.cuda.synchronize(device)
+            if dist:
+                dist.barrier()
+        total_ms = float(sum(step_ms))
+        if dist:
+            t = torch.tensor([total_ms], device=f"cuda:{device}")
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            total_ms = float(t.item())
+        value = world * n_cand * args.steps / (total_ms / 1e3)
+        feasible_frac = res["count"] / n_cand
+
+        # roofline of the scoring kernel: algorithmic FLOPs per launch / mean launch time
+        fpc = flops_per_candidate(prob)
+        per_launch_ms = float(sum(score_ms)) / max(score_launches, 1)
+        per_launch_flops = fpc * n_cand / (score_launches / args.steps)
+        peaks, src = _peaks()
+        achieved = per_launch_flops / (per_launch_ms / 1e3) / 1e12
+        if prec == "bf16":
+            peak = float(peaks["bf16_tflops_sustained"])
+            roof = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                    "frac": achieved / peak, "frac_burst": achieved / float(peaks["bf16_tflops"]),
+                    "peak_source": f"{src} bf16 sustained (burst {peaks['bf16_tflops']})"}
+        else:
+            sms = torch.cuda.get_device_properties(device).multi_processor_count
+            peak = sms * 128 * 2 * float(peaks.get("sm_max_mhz", 2070.0)) * 1e6 / 1e12
+            roof = {"bound": "alu", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                    "frac": achieved / peak,
+                    "peak_source": f"{sms} SMs x 128 FP32 lanes x 2 FLOP x {peaks.get('sm_max_mhz', 2070.0)} MHz"}
+        roof.update({"traffic": None, "kernel": "scoring kernel (one launch per 2^24 candidates)",
+                     "flops_per_candidate": fpc, "launch_ms": per_launch_ms})
+
+        # end to end through the C ABI from host buffers: create (uploads) + search + result
+        e2e_ms = []
+        for _ in range(max(2, min(args.steps, 5))):
+            torch.cuda.synchronize(device)
+            t0 = time.perf_counter()
+            with mf.Context(prob, device=device) as c2:
+                c2.search(K_TOP, chunk=CHUNK)
+                st2 = c2.stats()
+            e2e_ms.append(1e3 * (time.perf_counter() - t0))
+        e2e = {"value": n_cand / (statistics.median(e2e_ms) / 1e3), "unit": UNIT,
+               "h2d_bytes_per_step": int(st2["h2d_bytes_create"]),
+               "d2h_bytes_per_step": int(st2["d2h_bytes_last"]),
+               "how": "mf_create from host arrays + mf_search_exhaustive + mf_destroy, host wall clock, median"}
+
+    ga = ga_latency(mf, torch, device, args.ga_decisions) if rank == 0 else None
+    base = cpu_baseline(W.large(precision="fp32")) if (rank == 0 and world == 1 and not args.no_cpu) else None
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if prec == "bf16" else "f32",
+                "data": "synthetic", "config": workload_config(prec), "roofline": roof,
+                "cpu_baseline": base, "e2e": e2e, "gpu_launches": launches, "clocks": clk.summary(),
+                "feasible_fraction": feasible_frac, "best": {"idx": res["best_idx"], "J": res["best_score"],
+                                                             "count": res["count"]},
+                "ga": ga}
+        print(json.dumps(line), flush=True)
+    if dist:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--precision", default=os.environ.get("MF_BENCH_PRECISION", "bf16"),
+                    choices=["bf16", "fp32"])
+    ap.add_argument("--ga-decisions", type=int, default=10)
+    ap.add_argument("--no-cpu", action="store_true", help="skip the CPU-baseline leg")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -111,6 +111,19 @@ typedef struct {
   int32_t elitism;             /* 0 or 1 */
 } mf_ga_params;
 
+/* Instrumentation of the last calls on a context (host-side bookkeeping plus
+ * CUDA events recorded on the call's stream; no extra synchronisation). */
+typedef struct {
+  uint64_t h2d_bytes_create;   /* bytes mf_create copied host -> device */
+  uint64_t d2h_bytes_last;     /* bytes the last synchronous call copied device -> host */
+  int32_t kernel_launches_last;/* library kernels launched by the last search / GA run */
+  int32_t score_launches_last; /* of which scoring launches (one per chunk) */
+  float score_ms_last;         /* device time from the first to the end of the last scoring
+                                  launch of the last search */
+  float total_ms_last;         /* device time of the whole last search (scoring, merge,
+                                  re-scoring, result copy) */
+} mf_stats;
+
 /* Name of a status code (static string). */
 const char *mf_status_string(mf_status s);
 
@@ -189,6 +202,9 @@ mf_status mf_ga_step(mf_ctx *ctx, const mf_ga_params *g, uint64_t seed, int32_t 
  * fitness.  Synchronous. */
 mf_status mf_ga_run(mf_ctx *ctx, const mf_ga_params *g, uint64_t seed, int32_t *best_genome,
                     float *best_fitness, void *stream);
+
+/* Read the context's instrumentation (see mf_stats). */
+mf_status mf_get_stats(const mf_ctx *ctx, mf_stats *out);
 
 /* Synchronise `stream`, then return MF_EDEVICE if any asynchronous call since the
  * last check saw an invalid index or gene (and clear that flag), else MF_OK. */

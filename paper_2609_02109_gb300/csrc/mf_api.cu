@@ -78,6 +78,8 @@ static void free_ctx(mf_ctx* c) {
   cudaFree(c->d_ga_out);
   if (c->ga_exec) cudaGraphExecDestroy(c->ga_exec);
   if (c->cap_stream) cudaStreamDestroy(c->cap_stream);
+  for (int j = 0; j < 3; ++j)
+    if (c->ev[j]) cudaEventDestroy(c->ev[j]);
   if (c->h_stage) cudaFreeHost(c->h_stage);
   delete c;
 }
@@ -227,11 +229,14 @@ mf_status mf_create(const mf_problem* p, mf_ctx** out) {
       (e = upload((void**)&c->d_w32, w32.data(), sizeof(float) * w32.size())) != cudaSuccess ||
       (e = upload((void**)&c->d_wT, wT.data(), sizeof(float) * wT.size())) != cudaSuccess ||
       (e = cudaMalloc((void**)&c->d_status, sizeof(uint32_t))) != cudaSuccess ||
-      (e = cudaMemset(c->d_status, 0, sizeof(uint32_t))) != cudaSuccess) {
+      (e = cudaMemset(c->d_status, 0, sizeof(uint32_t))) != cudaSuccess ||
+      (e = cudaEventCreate(&c->ev[0])) != cudaSuccess || (e = cudaEventCreate(&c->ev[1])) != cudaSuccess ||
+      (e = cudaEventCreate(&c->ev[2])) != cudaSuccess) {
     mf_status st2 = cuda_fail(e, "mf_create upload");
     free_ctx(c);
     return st2;
   }
+  c->stats.h2d_bytes_create = sizeof(float) * ((size_t)sumK * p->d_local + dem4.size() + w32.size() + wT.size());
   P.x = c->d_x;
   P.dem = c->d_dem;
   P.w32 = c->d_w32;
@@ -352,6 +357,8 @@ mf_status mf_search_range(mf_ctx* ctx, uint64_t lo, uint64_t hi, int32_t k, uint
   unsigned long long* cnt = (unsigned long long*)(base + o_cnt);
   MF_CUDA(cudaMemsetAsync(cnt, 0, sizeof(unsigned long long), s));
 
+  int launches = 0, score_launches = 0;
+  MF_CUDA(cudaEventRecord(ctx->ev[0], s));
   RangeArgs a{};
   a.k = kcap;
   a.lists_s = ls;
@@ -364,6 +371,8 @@ mf_status mf_search_range(mf_ctx* ctx, uint64_t lo, uint64_t hi, int32_t k, uint
     a.len = 0;
     st = tc ? tc_search_chunk(ctx, a, s) : f32_search_chunk(ctx, a, s);
     if (st != MF_OK) return st;
+    ++launches;
+    ++score_launches;
   }
   for (uint64_t b = lo; b < hi; b += chunk) {
     a.base = b;
@@ -371,14 +380,19 @@ mf_status mf_search_range(mf_ctx* ctx, uint64_t lo, uint64_t hi, int32_t k, uint
     st = tc ? tc_search_chunk(ctx, a, s) : f32_search_chunk(ctx, a, s);
     if (st != MF_OK) return st;
     a.first = 0;
+    ++launches;
+    ++score_launches;
   }
+  MF_CUDA(cudaEventRecord(ctx->ev[1], s));
   st = merge_lists(ctx, ls, li, grid, kcap, ts, ti, ms, mi, s);
+  ++launches;
   if (st != MF_OK) return st;
   if (tc) {
     // exact fp32 re-scoring of the tensor-core shortlist, then the final top-k
     st = f32_score_list_ex(ctx, mi, kcap, rs, rp, s);
     if (st != MF_OK) return st;
     st = select_topk(ctx, rs, mi, kcap, k, fs, fi, s);
+    launches += 3;
   } else {
     MF_CUDA(cudaMemcpyAsync(fs, ms, sizeof(float) * k, cudaMemcpyDeviceToDevice, s));
     MF_CUDA(cudaMemcpyAsync(fi, mi, sizeof(uint64_t) * k, cudaMemcpyDeviceToDevice, s));
@@ -396,8 +410,14 @@ mf_status mf_search_range(mf_ctx* ctx, uint64_t lo, uint64_t hi, int32_t k, uint
   MF_CUDA(cudaMemcpyAsync(h_i, fi, sizeof(uint64_t) * k, cudaMemcpyDeviceToHost, s));
   MF_CUDA(cudaMemcpyAsync(h_s, fs, sizeof(float) * k, cudaMemcpyDeviceToHost, s));
   MF_CUDA(cudaMemcpyAsync(h_c, cnt, sizeof(unsigned long long), cudaMemcpyDeviceToHost, s));
+  MF_CUDA(cudaEventRecord(ctx->ev[2], s));
   st = read_status(ctx, s, h_status, true);
   if (st != MF_OK) return st;
+  ctx->stats.kernel_launches_last = launches;
+  ctx->stats.score_launches_last = score_launches;
+  ctx->stats.d2h_bytes_last = (sizeof(uint64_t) + sizeof(float)) * k + sizeof(unsigned long long) + sizeof(uint32_t);
+  MF_CUDA(cudaEventElapsedTime(&ctx->stats.score_ms_last, ctx->ev[0], ctx->ev[1]));
+  MF_CUDA(cudaEventElapsedTime(&ctx->stats.total_ms_last, ctx->ev[0], ctx->ev[2]));
   if (*h_status & kStatusTimeout) {
     g_last_error = "a bounded device wait gave up";
     return MF_ETIMEOUT;
@@ -480,6 +500,14 @@ mf_status mf_ga_run(mf_ctx* ctx, const mf_ga_params* g, uint64_t seed, int32_t* 
   if (st != MF_OK) return st;
   std::memcpy(best_genome, h_g, sizeof(int32_t) * N);
   *best_fitness = *h_f;
+  ctx->stats.d2h_bytes_last = sizeof(int32_t) * N + sizeof(float) + sizeof(uint32_t);
+  ctx->stats.kernel_launches_last = 2 + g->gens * 2 + (g->gens - 1);  // init, (wide + combine) x gens, steps, best
+  return MF_OK;
+}
+
+mf_status mf_get_stats(const mf_ctx* ctx, mf_stats* out) {
+  if (!ctx || !out) return einval("NULL argument");
+  *out = ctx->stats;
   return MF_OK;
 }
 

@@ -192,6 +192,9 @@ struct mf_ctx {
   uint64_t params_version = 0;
   uint64_t ga_version = ~0ull;
   mf_ga_params ga_key{};
+  // instrumentation
+  mf_stats stats{};
+  cudaEvent_t ev[3] = {nullptr, nullptr, nullptr};
 };
 
 namespace mf {

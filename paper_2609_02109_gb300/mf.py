@@ -23,7 +23,8 @@ EMPTY = (1 << 64) - 1
 
 _EXPORTS = ["mf_status_string", "mf_last_error", "mf_create", "mf_destroy", "mf_space_size",
             "mf_set_objective", "mf_score_batch", "mf_search_range", "mf_search_exhaustive",
-            "mf_ga_generation", "mf_ga_init", "mf_ga_step", "mf_ga_run", "mf_check_device_status"]
+            "mf_ga_generation", "mf_ga_init", "mf_ga_step", "mf_ga_run", "mf_check_device_status",
+            "mf_get_stats"]
 
 
 class MFError(RuntimeError):
@@ -47,6 +48,12 @@ class _Problem(C.Structure):
 class _Result(C.Structure):
     _fields_ = [("best_idx", C.c_uint64), ("best_score", C.c_float), ("feasible_count", C.c_uint64),
                 ("k", C.c_int32), ("topk_idx", C.c_void_p), ("topk_score", C.c_void_p)]
+
+
+class _Stats(C.Structure):
+    _fields_ = [("h2d_bytes_create", C.c_uint64), ("d2h_bytes_last", C.c_uint64),
+                ("kernel_launches_last", C.c_int32), ("score_launches_last", C.c_int32),
+                ("score_ms_last", C.c_float), ("total_ms_last", C.c_float)]
 
 
 class _GAParams(C.Structure):
@@ -73,6 +80,7 @@ def _load() -> C.CDLL:
     lib.mf_ga_step.argtypes = [vp, C.POINTER(_GAParams), u64, i32, vp, vp, vp, vp]
     lib.mf_ga_run.argtypes = [vp, C.POINTER(_GAParams), u64, vp, vp, vp]
     lib.mf_check_device_status.argtypes = [vp, vp]
+    lib.mf_get_stats.argtypes = [vp, C.POINTER(_Stats)]
     for name in _EXPORTS[2:]:
         getattr(lib, name).restype = st
     return lib
@@ -218,6 +226,11 @@ class Context:
         _check(_lib.mf_ga_run(self._h, C.byref(g), int(seed), genome.ctypes.data, C.byref(fit),
                               _stream(self.device)), "mf_ga_run")
         return float(fit.value), genome
+
+    def stats(self) -> dict:
+        st = _Stats()
+        _check(_lib.mf_get_stats(self._h, C.byref(st)), "mf_get_stats")
+        return {f: getattr(st, f) for f, _ in _Stats._fields_}
 
     def check_status(self) -> int:
         """MF_OK, or the status of the first device-reported problem (clears it)."""
