@@ -206,6 +206,38 @@ mf_status mf_ga_run(mf_ctx *ctx, const mf_ga_params *g, uint64_t seed, int32_t *
 /* Read the context's instrumentation (see mf_stats). */
 mf_status mf_get_stats(const mf_ctx *ctx, mf_stats *out);
 
+/* Exhaustive search without any device allocation.
+ *
+ * The paper has no counterpart to this call; it exists for callers that cannot
+ * call cudaMalloc -- for example a serving process whose memory pool has already
+ * claimed the device's memory, or a per-decision control loop that must not pay
+ * cudaMalloc's implicit device synchronisation.  It runs the exact fp32 search of
+ * mf_search_exhaustive on the problem `p` (host arrays, as for mf_create;
+ * precision must be MF_FP32) and fills `out` (host memory) the same way, without
+ * creating a context.  All device memory it uses -- a copy of the problem's
+ * tables and weights, the per-CTA running top-k lists, the merge buffers, the
+ * feasible counter and the status word -- lives in one fixed array of
+ * MF_NOALLOC_SCRATCH_BYTES that the library declares in device memory; every GPU
+ * that loads the library holds that array until the process exits.  The call
+ * allocates nothing (no cudaMalloc, cudaFree or other allocating routine).
+ *
+ * Limits (MF_EINVAL with a message beyond them): k <= MF_NOALLOC_MAX_TOPK, packed
+ * predictor weights <= MF_NOALLOC_MAX_WEIGHT_BYTES, and the whole layout within
+ * MF_NOALLOC_SCRATCH_BYTES.  At most MF_NOALLOC_MAX_CTAS CTAs are launched.
+ *
+ * The first call on a device looks up the array's device address (once per
+ * device, with that device current); make that first call before any stream
+ * capture.  Every call on a device shares the one array and overwrites it
+ * (what must start at zero is cleared at the start of each call), so calls
+ * that overlap on the GPU -- from several host threads or streams -- race and
+ * must be serialised by the caller.  Synchronous: returns after `out` is filled. */
+#define MF_NOALLOC_SCRATCH_BYTES (4u << 20)
+#define MF_NOALLOC_MAX_TOPK 64
+#define MF_NOALLOC_MAX_CTAS 256
+#define MF_NOALLOC_MAX_WEIGHT_BYTES (1u << 20)
+mf_status mf_search_exhaustive_noalloc(const mf_problem *p, int32_t k, uint64_t chunk,
+                                       mf_result *out, void *stream);
+
 /* Synchronise `stream`, then return MF_EDEVICE if any asynchronous call since the
  * last check saw an invalid index or gene (and clear that flag), else MF_OK. */
 mf_status mf_check_device_status(mf_ctx *ctx, void *stream);

@@ -604,3 +604,20 @@ mf_status f32_score_list(mf_ctx* c, const uint64_t* idx, const int32_t* genes, u
 }
 
 }  // namespace mf
+
+namespace mf {
+
+// Range-mode launch from a bare parameter block (no context): sets the kernel's
+// shared-memory limit and launches one chunk on `grid` CTAs.
+mf_status f32_search_chunk_params(const Params& P, int grid, const RangeArgs& a, cudaStream_t s) {
+  bool res;
+  const size_t smem = f32_smem_bytes(P, a.k, res);
+  ScoreFn fn = pick_fn(kModeRange, fixed_shape_id(P), res);
+  MF_CUDA(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024));
+  ListArgs L{};
+  fn<<<grid, kScoreThreads, smem, s>>>(P, a, L);
+  MF_CUDA(cudaGetLastError());
+  return MF_OK;
+}
+
+}  // namespace mf

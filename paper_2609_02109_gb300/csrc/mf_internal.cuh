@@ -227,6 +227,7 @@ size_t f32_smem_bytes(const Params& P, int k, bool& resident);
 int f32_grid(const mf_ctx* c);
 mf_status f32_prepare(mf_ctx* c);
 mf_status f32_search_chunk(mf_ctx* c, const RangeArgs& a, cudaStream_t s);
+mf_status f32_search_chunk_params(const Params& P, int grid, const RangeArgs& a, cudaStream_t s);
 mf_status f32_score_list(mf_ctx* c, const uint64_t* idx, const int32_t* genes, uint64_t n,
                          float* score, uint8_t* feas, float* pred, cudaStream_t s);
 // Exact re-scoring of a shortlist that may contain empty slots (index UINT64_MAX),

@@ -24,7 +24,7 @@ EMPTY = (1 << 64) - 1
 _EXPORTS = ["mf_status_string", "mf_last_error", "mf_create", "mf_destroy", "mf_space_size",
             "mf_set_objective", "mf_score_batch", "mf_search_range", "mf_search_exhaustive",
             "mf_ga_generation", "mf_ga_init", "mf_ga_step", "mf_ga_run", "mf_check_device_status",
-            "mf_get_stats"]
+            "mf_get_stats", "mf_search_exhaustive_noalloc"]
 
 
 class MFError(RuntimeError):
@@ -81,6 +81,7 @@ def _load() -> C.CDLL:
     lib.mf_ga_run.argtypes = [vp, C.POINTER(_GAParams), u64, vp, vp, vp]
     lib.mf_check_device_status.argtypes = [vp, vp]
     lib.mf_get_stats.argtypes = [vp, C.POINTER(_Stats)]
+    lib.mf_search_exhaustive_noalloc.argtypes = [C.POINTER(_Problem), i32, u64, C.POINTER(_Result), vp]
     for name in _EXPORTS[2:]:
         getattr(lib, name).restype = st
     return lib
@@ -109,6 +110,42 @@ def _ga(params: dict) -> _GAParams:
 
 def _f32(a) -> np.ndarray:
     return np.ascontiguousarray(a, dtype=np.float32)
+
+
+def _problem_struct(prob: dict, device: int, prec: str):
+    """mf_problem for a workload dict; returns (struct, arrays kept alive)."""
+    keep = {
+        "n_options": np.ascontiguousarray(prob["n_options"], dtype=np.int32),
+        "local_feats": _f32(prob["local_feats"]), "demand": _f32(prob["demand"]),
+        "weights": _f32(prob["weights"]),
+        "agg_scale": None if prob.get("agg_scale") is None else _f32(prob["agg_scale"]),
+        "sla": _f32(prob["sla"]), "obj_w": _f32(prob["obj_w"]),
+    }
+    ptr = lambda a: None if a is None else a.ctypes.data  # noqa: E731
+    k = keep
+    p = _Problem(int(k["n_options"].size), ptr(k["n_options"]), int(prob["d_local"]),
+                 int(prob["hidden1"]), int(prob["hidden2"]), ptr(k["local_feats"]), ptr(k["demand"]),
+                 ptr(k["weights"]), ptr(k["agg_scale"]), ptr(k["sla"]), ptr(k["obj_w"]),
+                 float(prob["vram_cap"]), float(prob.get("soft_penalty", 0.0)),
+                 1 if prob.get("out_act", "identity") == "sigmoid" else 0,
+                 1 if prob.get("objective", "weighted_thr") == "soft_lat" else 0,
+                 MF_BF16 if prec == "bf16" else MF_FP32, int(device))
+    return p, keep
+
+
+def search_exhaustive_noalloc(prob: dict, k: int, chunk: int = 0, device: int | None = None) -> dict:
+    """mf_search_exhaustive_noalloc: the exact fp32 search with no device allocation
+    (all device memory in the library's fixed array); same result fields as
+    Context.search."""
+    device = torch.cuda.current_device() if device is None else int(device)
+    p, _keep = _problem_struct(prob, device, "fp32")
+    ti = np.empty(k, dtype=np.uint64)
+    ts = np.empty(k, dtype=np.float32)
+    r = _Result(0, 0.0, 0, k, ti.ctypes.data, ts.ctypes.data)
+    _check(_lib.mf_search_exhaustive_noalloc(C.byref(p), int(k), int(chunk), C.byref(r),
+                                              _stream(device)), "mf_search_exhaustive_noalloc")
+    return dict(best_idx=int(r.best_idx), best_score=float(r.best_score),
+                count=int(r.feasible_count), topk_idx=ti, topk_score=ts)
 
 
 class Context:
