@@ -72,7 +72,7 @@ static double relu(double v) { return v < 0.0 ? 0.0 : v; }
  * identity, so the layers are Linear -> ReLU -> [Linear -> ReLU] -> Linear,
  * with an optional sigmoid on the two outputs (the paper's output unit). */
 static void predictor(const orc_problem *p, int32_t model, const double *z,
-                      double *thr, double *lat) {
+                      double *thr, double *lat, double *mag) {
   const int32_t din = d_in_of(p), h1 = p->hidden1, h2 = p->hidden2;
   const float *w = p->weights + (int64_t)model * params_per_model(p);
   const float *W1 = w;
@@ -104,9 +104,14 @@ static void predictor(const orc_problem *p, int32_t model, const double *z,
   double y[2];
   for (int32_t o = 0; o < 2; ++o) {
     double s = (double)b3[o];
-    for (int32_t k = 0; k < hl; ++k) s += (double)W3[(int64_t)o * hl + k] * h[k];
+    double m = fabs((double)b3[o]);
+    for (int32_t k = 0; k < hl; ++k) {
+      s += (double)W3[(int64_t)o * hl + k] * h[k];
+      m += fabs((double)W3[(int64_t)o * hl + k]) * fabs(h[k]);
+    }
     if (p->out_act == 1) s = 1.0 / (1.0 + exp(-s));
     y[o] = s;
+    if (mag) mag[o] = m;
   }
   *thr = y[0];
   *lat = y[1];
@@ -144,7 +149,7 @@ double orc_score_digits(const orc_problem *p, const int32_t *o, int32_t *feasibl
     for (int32_t k = 0; k < dl; ++k) z[k] = (double)x[k];
     for (int c = 0; c < 4; ++c) z[dl + c] = A[c] * s[c];
     double thr, lat;
-    predictor(p, i, z, &thr, &lat);
+    predictor(p, i, z, &thr, &lat, NULL);
     if (pred) { pred[2 * i] = thr; pred[2 * i + 1] = lat; }
     /* Eq. 3 first term, with the throughput-weighted objective sum_i w_i thr_i */
     J += (double)p->obj_w[i] * thr;
@@ -186,6 +191,54 @@ void orc_score_list(const orc_problem *p, const uint64_t *idx, uint64_t n,
     }
     score[t] = J;
     if (feasible) feasible[t] = f;
+  }
+}
+
+/* Condition scale of every predictor output of one candidate: the magnitude
+ * |b3_o| + sum_k |W3[o][k]| |h_k| of the terms of the final dot product, with
+ * the exact last hidden layer h (before the output activation).  Rounding
+ * errors of a reduced-precision evaluation scale with this sum, not with the
+ * possibly cancelling output itself. */
+static void pred_scale_digits(const orc_problem *p, const int32_t *o, double *scale) {
+  const int32_t n = p->n_models, dl = p->d_local, din = d_in_of(p);
+  double A[4] = {0.0, 0.0, 0.0, (double)n};
+  for (int32_t i = 0; i < n; ++i) {
+    const float *d = p->demand + 3 * (option_offset(p, i) + o[i]);
+    A[0] += (double)d[0]; A[1] += (double)d[1]; A[2] += (double)d[2];
+  }
+  double s[4];
+  if (p->agg_scale) {
+    for (int c = 0; c < 4; ++c) s[c] = (double)p->agg_scale[c];
+  } else {
+    s[0] = 1.0 / (0.6 * n); s[1] = 1.0 / (20.0 * n); s[2] = 1.0 / (1500.0 * n); s[3] = 1.0 / 8.0;
+    for (int c = 0; c < 4; ++c) s[c] = (double)(float)s[c];
+  }
+  double z[din];
+  for (int32_t i = 0; i < n; ++i) {
+    const float *x = p->local_feats + (int64_t)dl * (option_offset(p, i) + o[i]);
+    for (int32_t k = 0; k < dl; ++k) z[k] = (double)x[k];
+    for (int c = 0; c < 4; ++c) z[dl + c] = A[c] * s[c];
+    double thr, lat;
+    predictor(p, i, z, &thr, &lat, scale + 2 * i);
+  }
+}
+
+void orc_pred_scale_list(const orc_problem *p, const uint64_t *idx, uint64_t n, double *scale,
+                         int32_t nthreads) {
+  const uint64_t total = orc_space_size(p);
+  const int32_t nm = p->n_models;
+  (void)nthreads;
+#ifdef _OPENMP
+#pragma omp parallel for schedule(static) num_threads(nthreads > 0 ? nthreads : 1)
+#endif
+  for (int64_t t = 0; t < (int64_t)n; ++t) {
+    int32_t o[64];
+    if (idx[t] < total) {
+      orc_decode(p, idx[t], o);
+      pred_scale_digits(p, o, scale + 2 * nm * t);
+    } else {
+      for (int32_t j = 0; j < 2 * nm; ++j) scale[2 * nm * t + j] = 0.0;
+    }
   }
 }
 

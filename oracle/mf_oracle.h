@@ -8,6 +8,7 @@
  *
  * Parity status per function (pins live in tests/test_oracle_*.py):
  *   orc_space_size, orc_decode        pinned (Eq. 1 sizes, numpy.unravel_index)
+ *   orc_pred_scale_list               pinned (equals |output| in the linear case)
  *   orc_score_digits                  pinned (hand example, linear case,
  *                                     aggregate invariant, separable closed form,
  *                                     sigmoid closed form, soft-penalty hand value)
@@ -59,6 +60,12 @@ double orc_score_digits(const orc_problem *p, const int32_t *o, int32_t *feasibl
 void orc_score_list(const orc_problem *p, const uint64_t *idx, uint64_t n,
                     double *score, int32_t *feasible, double *pred, double *agg,
                     int32_t nthreads);
+
+/* Per candidate and model, the condition scale of each predictor output:
+ * |b3_o| + sum_k |W3[o][k]| |h_k| with the exact last hidden layer h.
+ * scale: [n][N][2]. */
+void orc_pred_scale_list(const orc_problem *p, const uint64_t *idx, uint64_t n, double *scale,
+                         int32_t nthreads);
 
 /* Exhaustive search over [lo, hi): top-k by (J desc, idx asc) and the feasible
  * count.  Unfilled slots are (UINT64_MAX, -inf). */

@@ -68,6 +68,8 @@ def _load():
             lib.orc_score_digits.argtypes = [P, vp, vp, vp, vp]; lib.orc_score_digits.restype = dbl
             lib.orc_score_list.argtypes = [P, vp, u64, vp, vp, vp, vp, i32]
             lib.orc_score_list.restype = None
+            lib.orc_pred_scale_list.argtypes = [P, vp, u64, vp, i32]
+            lib.orc_pred_scale_list.restype = None
             lib.orc_exhaustive.argtypes = [P, u64, u64, i32, vp, vp, vp, i32]
             lib.orc_exhaustive.restype = None
             lib.orc_splitmix64.argtypes = [u64, u64]; lib.orc_splitmix64.restype = u64
@@ -140,6 +142,13 @@ class Oracle:
         if with_pred:
             return score, feas.astype(bool), pred, agg
         return score, feas.astype(bool)
+
+    def pred_scale(self, idx) -> np.ndarray:
+        """[n][N][2] condition scales |b3| + sum_k |W3_k||h_k| of the outputs."""
+        idx = np.ascontiguousarray(idx, dtype=np.uint64)
+        out = np.empty((idx.size, self.n, 2), dtype=np.float64)
+        self.lib.orc_pred_scale_list(C.byref(self.p), _ptr(idx), idx.size, _ptr(out), self.nthreads)
+        return out
 
     def exhaustive(self, k: int, lo: int = 0, hi: int | None = None, nthreads: int | None = None):
         hi = self.space_size() if hi is None else hi

@@ -1,23 +1,709 @@
-// Tensor-core (tcgen05, bf16) scorer -- placeholder until the kernel lands.
+// Tensor-core (tcgen05, bf16 x bf16 -> fp32) scorer for sm_103a.
+//
+// Same computation as the exact fp32 path (arXiv 2609.02109: Eq. 1 decode, the
+// aggregate GPU state, the per-model MeanField MLP of Eq. 6, the constraints of
+// Eq. 4 and the objective of Eq. 3), with the MLP layers run as UMMA tiles:
+//
+//   layer 1   D1[128 x h1]  = A1[128 x k1] . B1^T    A1 = [x_i | agg hi | 1 | agg lo]
+//   layer 2   D2[128 x h2]  = H1[128 x h1] . W2^T    (+ b2, ReLU in the epilogue)
+//   layer 3   D3[128 x n3] += H2[128 x h2] . B3_i^T  B3_i puts W3_i's two rows in
+//                                                    columns i (thr) and n3/2 + i (lat),
+//                                                    so D3 accumulates all N models.
+//
+// One persistent CTA per SM runs up to four independent 128-row pipelines of
+// four warps each (warp q of a pipeline owns TMEM lanes 32q..32q+31).  Each
+// pipeline keeps every A operand in tensor memory (layer inputs written with
+// tcgen05.st, hidden activations converted in place from the fp32 accumulators
+// with cvt.rn.relu.bf16x2), so the tensor core reads only the weights (B) from
+// shared memory.  The weights are staged once per CTA with one TMA bulk copy.
+// The pipeline's first thread issues the MMAs and commits them to an mbarrier
+// that the pipeline's threads wait on (bounded; a wait that gives up raises the
+// status word and the kernel runs to completion without further waits).
+//
+// Biases: b1 rides in A1's constant-1 column, b2 is added in the layer-2
+// epilogue, b3 in the final epilogue.  The aggregate enters layer 1 as a bf16
+// hi/lo pair (two columns per component with the same weight), so its rounding
+// error is ~2^-16 rather than 2^-9.
+#include <cuda_bf16.h>
+
+#include <cstring>
+#include <vector>
+
 #include "mf_internal.cuh"
 
 namespace mf {
 
+// ---------------------------------------------------------------------------
+// PTX wrappers (tcgen05 / mbarrier / bulk copy), written from the PTX ISA.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          smem_u32(dst)),
+      "l"(src), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+__device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+
+__device__ __forceinline__ void named_bar(int id, int nthreads) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+
+// OR of `pred` over the threads of a named barrier (also a barrier).
+__device__ __forceinline__ bool named_bar_or(int id, int nthreads, bool pred) {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred pi, po;\n setp.ne.u32 pi, %1, 0;\n bar.red.or.pred po, %2, %3, pi;\n"
+      " selp.u32 %0, 1, 0, po;\n}"
+      : "=r"(r)
+      : "r"((uint32_t)pred), "r"(id), "r"(nthreads)
+      : "memory");
+  return r != 0;
+}
+
+// UMMA shared-memory descriptor: K-major, no swizzle.  lbo = byte distance of
+// core matrices adjacent in K, sbo = byte distance of adjacent 8-row groups.
+__device__ __forceinline__ uint64_t smem_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)((lbo >> 4) & 0x3FFFu) << 16) |
+         ((uint64_t)((sbo >> 4) & 0x3FFFu) << 32) | (1ull << 46);
+}
+
+// Instruction descriptor of kind::f16: bf16 A and B (K-major), fp32 D, M = 128.
+__host__ __device__ constexpr uint32_t idesc_bf16(int n) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
+}
+
+// D[tmem] (+)= A[tmem] . B[smem]^T, one 128 x n x 16 MMA.
+__device__ __forceinline__ void mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                                       uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                   smem_u32(bar))
+               : "memory");
+}
+
+// ReLU then round to bf16, two values per register: `lo` in the low half.
+__device__ __forceinline__ uint32_t relu_bf16x2(uint32_t lo, uint32_t hi) {
+  uint32_t d;
+  asm("cvt.rn.relu.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(__uint_as_float(hi)), "f"(__uint_as_float(lo)));
+  return d;
+}
+
+__device__ __forceinline__ uint32_t bf16_bits(float v) {
+  return (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v));
+}
+
+__device__ __forceinline__ void tmem_ld_x16(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+               : "r"(taddr));
+}
+
+__device__ __forceinline__ void tmem_ld_x32(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+               : "r"(taddr));
+}
+
+__device__ __forceinline__ void tmem_st_x8(uint32_t taddr, const uint32_t (&v)[8]) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};"
+               :: "r"(taddr), "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7])
+               : "memory");
+}
+
+__device__ __forceinline__ void tmem_st_x16(uint32_t taddr, const uint32_t (&v)[16]) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};"
+               :: "r"(taddr), "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
+               : "memory");
+}
+
+
+// ---------------------------------------------------------------------------
+// The kernel
+// ---------------------------------------------------------------------------
+enum { kTcRange = 0, kTcList = 1 };
+constexpr int kTcMaxPipes = 4;
+constexpr uint32_t kWaitLimit = 1u << 26;
+
+struct TcList {
+  const uint64_t* idx;
+  uint64_t n;
+  float* score;
+  uint8_t* feas;
+  float* pred;
+};
+
+struct PipeWait {
+  volatile int* abort;
+  uint32_t* status;
+  // Bounded wait for `parity` of `bar`; on giving up flags the status word and
+  // makes every later wait return at once.
+  __device__ __forceinline__ void operator()(uint64_t* bar, uint32_t parity) const {
+    uint32_t n = 0;
+    while (!*abort) {
+      if (mbar_try_wait(bar, parity)) return;
+      if (++n > kWaitLimit) {
+        *abort = 1;
+        atomicOr(status, kStatusTimeout);
+        return;
+      }
+    }
+  }
+};
+
+template <int MODE>
+__global__ void __launch_bounds__(kTcMaxPipes * 128, 1)
+k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
+  extern __shared__ __align__(1024) unsigned char smem[];
+  __shared__ uint32_t s_tmem;
+  __shared__ int s_abort;
+  const int tid = threadIdx.x;
+  const int warp = tid >> 5, lane = tid & 31;
+  const int pipe = warp >> 2, wq = warp & 3;
+  const int row = wq * 32 + lane;
+  const int N = P.n_models;
+  const int npipes = T.pipes;
+
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + T.sm_bar);
+  uint32_t* xw_s = reinterpret_cast<uint32_t*>(smem + T.sm_xw);
+  float4* dem_s = reinterpret_cast<float4*>(smem + T.sm_dem);
+  float* b2_s = reinterpret_cast<float*>(smem + T.sm_b2);
+  float* b3_s = reinterpret_cast<float*>(smem + T.sm_b3);
+
+  if (tid == 0) {
+    s_abort = 0;
+    for (int j = 0; j <= npipes; ++j) mbar_init(&bars[j], 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&s_tmem)),
+                 "r"(512)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  __syncthreads();
+  if (tid == 0) {
+    // weights: one TMA bulk copy per 32 KB piece, all completing on bars[0]
+    mbar_arrive_expect_tx(&bars[0], T.img_bytes);
+    for (uint32_t o = 0; o < T.img_bytes; o += 32768u) {
+      const uint32_t b = T.img_bytes - o < 32768u ? T.img_bytes - o : 32768u;
+      bulk_g2s(smem + o, static_cast<const unsigned char*>(T.img) + o, b, &bars[0]);
+    }
+  }
+  // option tables and biases with ordinary loads
+  const int sumK = P.off[N - 1] + P.K[N - 1];
+  for (int e = tid; e < sumK * T.kw; e += blockDim.x) xw_s[e] = T.xw[e];
+  for (int e = tid; e < sumK; e += blockDim.x) dem_s[e] = P.dem[e];
+  for (int e = tid; e < N * T.h2; e += blockDim.x) b2_s[e] = T.b2[e];
+  for (int e = tid; e < 2 * N; e += blockDim.x) b3_s[e] = T.b3[e];
+
+  // per-pipeline running top-k (range mode)
+  CtaTopK tk{};
+  const int kcap = R.k;
+  if (MODE == kTcRange) {
+    unsigned char* q = smem + T.sm_topk +
+                       (size_t)pipe * ((sizeof(uint64_t) + sizeof(float)) * (2 * (size_t)kcap + 128) + 16);
+    tk.li = reinterpret_cast<uint64_t*>(q); q += sizeof(uint64_t) * kcap;
+    tk.ni = reinterpret_cast<uint64_t*>(q); q += sizeof(uint64_t) * kcap;
+    tk.qi = reinterpret_cast<uint64_t*>(q); q += sizeof(uint64_t) * 128;
+    tk.ls = reinterpret_cast<float*>(q); q += sizeof(float) * kcap;
+    tk.ns = reinterpret_cast<float*>(q); q += sizeof(float) * kcap;
+    tk.qs = reinterpret_cast<float*>(q); q += sizeof(float) * 128;
+    tk.qn = reinterpret_cast<int*>(q);
+    tk.k = kcap;
+    const size_t gl = ((size_t)blockIdx.x * npipes + pipe) * kcap;
+    for (int e = row; e < kcap; e += 128) {
+      tk.ls[e] = R.first ? -INFINITY : R.lists_s[gl + e];
+      tk.li[e] = R.first ? kEmptyIdx : R.lists_i[gl + e];
+    }
+    if (row == 0) *tk.qn = 0;
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = s_tmem;
+  const PipeWait wait_bar{&s_abort, P.status};
+  wait_bar(&bars[0], 0);  // weights landed
+
+  const uint32_t tp = tmem + (uint32_t)(pipe * T.pipe_stride);
+  const uint32_t lane_off = (uint32_t)(wq * 32) << 16;
+  const uint32_t tD = tp + T.col_d, tH = tp + T.col_h, tA = tp + T.col_a, tD3 = tp + T.col_d3;
+  const bool leader = (wq == 0 && lane == 0);
+  uint64_t* mbar = &bars[1 + pipe];
+  uint32_t phase = 0;
+  const int barid = 1 + pipe;
+  const uint32_t smem_base = smem_u32(smem);
+  const uint32_t id1 = idesc_bf16(T.h1), id2 = idesc_bf16(T.h2), id3 = idesc_bf16(T.n3);
+  const uint32_t sbo1 = (uint32_t)(T.k1 / 8) * 128u, sbo2 = (uint32_t)(T.h1 / 8) * 128u,
+                 sbo3 = (uint32_t)(T.hl / 8) * 128u;
+  const float vcap = P.vram_cap;
+
+  float thr_s = -INFINITY;
+  uint64_t thr_i = kEmptyIdx;
+  if (MODE == kTcRange) {
+    named_bar(barid, 128);
+    thr_s = tk.ls[kcap - 1];
+    thr_i = tk.li[kcap - 1];
+  }
+  unsigned int my_count = 0;
+
+  const uint64_t n = MODE == kTcRange ? R.len : L.n;
+  const uint64_t gpipe = (uint64_t)blockIdx.x * npipes + pipe;
+  const uint64_t gstride = (uint64_t)gridDim.x * npipes;
+
+  auto issue_mma1 = [&](int i) {
+    const uint32_t b = smem_base + T.off_b1[i];
+    for (int s = 0; s < T.k1 / 16; ++s)
+      mma_ts(tD, tA + 8 * s, smem_desc(b + 256u * s, 128u, sbo1), id1, s > 0);
+  };
+  auto issue_mma2 = [&](int i) {
+    const uint32_t b = smem_base + T.off_b2[i];
+    for (int s = 0; s < T.h1 / 16; ++s)
+      mma_ts(tD, tH + 8 * s, smem_desc(b + 256u * s, 128u, sbo2), id2, s > 0);
+  };
+  auto issue_mma3 = [&](int i) {
+    const uint32_t b = smem_base + T.off_b3[i];
+    for (int s = 0; s < T.hl / 16; ++s)
+      mma_ts(tD3, tH + 8 * s, smem_desc(b + 256u * s, 128u, sbo3), id3, (i > 0 || s > 0));
+  };
+  // fp32 accumulators [cols c0, c0+32) -> (+ bias) -> ReLU -> bf16 pairs at H[c0/2 ..)
+  auto epilogue = [&](int width, const float* bias) {
+    for (int c0 = 0; c0 < width; c0 += 32) {
+      uint32_t r[32];
+      tmem_ld_x32(tD + lane_off + c0, r);
+      tmem_wait_ld();
+      if (bias) {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) r[j] = __float_as_uint(__uint_as_float(r[j]) + bias[c0 + j]);
+      }
+      uint32_t h[16];
+#pragma unroll
+      for (int j = 0; j < 16; ++j) h[j] = relu_bf16x2(r[2 * j], r[2 * j + 1]);
+      tmem_st_x16(tH + lane_off + (c0 >> 1), h);
+    }
+  };
+
+  for (uint64_t tile = gpipe; tile * 128 < n; tile += gstride) {
+    const uint64_t t = tile * 128 + row;
+    bool valid = t < n;
+    uint64_t idx = 0;
+    if (valid) idx = MODE == kTcRange ? R.base + t : L.idx[t];
+    if (MODE == kTcList && valid && idx >= P.total) {
+      atomicOr(P.status, kStatusBadInput);
+      valid = false;
+    }
+    if (!valid) idx = 0;  // compute on candidate 0, discard at the end
+    // aggregate state (fp32, model order) and its bf16 hi/lo words
+    float A0 = 0.f, A1 = 0.f, A2 = 0.f;
+    for (int i = 0; i < N; ++i) {
+      const float4 d = dem_s[P.off[i] + digit_of(P, idx, i)];
+      A0 += d.x; A1 += d.y; A2 += d.z;
+    }
+    uint32_t aw[4];
+    {
+      const float v0 = A0 * P.agg_scale[0], v1 = A1 * P.agg_scale[1], v2 = A2 * P.agg_scale[2];
+      const uint32_t h0 = bf16_bits(v0), h1 = bf16_bits(v1), h2 = bf16_bits(v2);
+      const uint32_t l0 = bf16_bits(v0 - __uint_as_float(h0 << 16));
+      const uint32_t l1 = bf16_bits(v1 - __uint_as_float(h1 << 16));
+      const uint32_t l2 = bf16_bits(v2 - __uint_as_float(h2 << 16));
+      aw[0] = h0 | (h1 << 16);
+      aw[1] = h2 | (0x3F80u << 16);  // bf16 1.0
+      aw[2] = l0 | (l1 << 16);
+      aw[3] = l2;
+    }
+    const int awo = T.dle >> 1;
+    auto write_a1 = [&](int i) {
+      const int r0 = (P.off[i] + digit_of(P, idx, i)) * T.kw;
+      // word j: local-feature pair, or aggregate word j - awo for awo <= j < awo + 4
+      auto word = [&](int j) -> uint32_t {
+        const int a = j - awo;
+        return a == 0 ? aw[0] : a == 1 ? aw[1] : a == 2 ? aw[2] : a == 3 ? aw[3] : xw_s[r0 + j];
+      };
+      if (T.kw == 8) {
+        uint32_t v[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) v[j] = word(j);
+        tmem_st_x8(tA + lane_off, v);
+      } else {
+        uint32_t v[16];
+#pragma unroll
+        for (int j = 0; j < 16; ++j) v[j] = word(j);
+        tmem_st_x16(tA + lane_off, v);
+      }
+    };
+
+    write_a1(0);
+    tmem_wait_st();
+    tc_fence_before();
+    named_bar(barid, 128);
+    for (int i = 0; i < N; ++i) {
+      if (leader) {
+        tc_fence_after();
+        if (i > 0) issue_mma3(i - 1);
+        issue_mma1(i);
+        mma_commit(mbar);
+      }
+      wait_bar(mbar, phase);
+      phase ^= 1u;
+      tc_fence_after();
+      epilogue(T.h1, nullptr);  // layer 1 (bias in the constant column)
+      if (T.h2 > 0) {
+        tmem_wait_st();
+        tc_fence_before();
+        named_bar(barid, 128);
+        if (leader) {
+          tc_fence_after();
+          issue_mma2(i);
+          mma_commit(mbar);
+        }
+        wait_bar(mbar, phase);
+        phase ^= 1u;
+        tc_fence_after();
+        epilogue(T.h2, b2_s + i * T.h2);  // layer 2
+      }
+      if (i + 1 < N) write_a1(i + 1);
+      tmem_wait_st();
+      tc_fence_before();
+      named_bar(barid, 128);
+    }
+    if (leader) {
+      tc_fence_after();
+      issue_mma3(N - 1);
+      mma_commit(mbar);
+    }
+    wait_bar(mbar, phase);
+    phase ^= 1u;
+    tc_fence_after();
+
+    // ---- final epilogue: per-model outputs, constraints, objective ----
+    uint32_t d3[32];
+    if (T.n3 == 16) {
+      uint32_t r16[16];
+      tmem_ld_x16(tD3 + lane_off, r16);
+      tmem_wait_ld();
+#pragma unroll
+      for (int j = 0; j < 16; ++j) d3[j] = r16[j];
+    } else {
+      tmem_ld_x32(tD3 + lane_off, d3);
+      tmem_wait_ld();
+    }
+    float J = 0.f, pen = 0.f;
+    bool sla_ok = true, sla_near = true;
+    const int half3 = T.n3 >> 1;  // thr of model i in column i, lat in column half3 + i
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      if (i >= N) break;
+      const float dthr = __uint_as_float(d3[i]);
+      const float dlat = __uint_as_float(half3 == 8 ? d3[(8 + i) & 31] : d3[(16 + i) & 31]);
+      const float thr = out_act(P, dthr + b3_s[2 * i]);
+      const float lat = out_act(P, dlat + b3_s[2 * i + 1]);
+      if (MODE == kTcList && valid && L.pred) {
+        L.pred[(t * N + i) * 2 + 0] = thr;
+        L.pred[(t * N + i) * 2 + 1] = lat;
+      }
+      J = fmaf(P.w[i], thr, J);
+      const float sla = P.sla[i];
+      sla_ok = sla_ok && (lat <= sla);
+      // shortlist test: within the bf16 error band of the ceiling
+      sla_near = sla_near && (lat <= sla + 2e-2f * fmaxf(fabsf(sla), fabsf(lat)));
+      const float over = lat - sla;
+      pen += over > 0.f ? over : 0.f;
+    }
+    bool feas = valid && A1 <= vcap;
+    bool cand = feas;
+    if (P.objective == MF_OBJ_WEIGHTED_THR) {
+      feas = feas && sla_ok;
+      cand = cand && sla_near;
+    } else {
+      J = fmaf(-P.soft_penalty, pen, J);
+    }
+    if (J != J) { feas = false; cand = false; }
+    if (MODE == kTcList) {
+      if (t < n) {
+        L.score[t] = feas ? J : -INFINITY;
+        if (L.feas) L.feas[t] = feas ? 1 : 0;
+      }
+    } else {
+      my_count += feas ? 1u : 0u;
+      const bool push = cand && precedes(J, idx, thr_s, thr_i);
+      if (push) {
+        const int pos = atomicAdd(tk.qn, 1);
+        tk.qs[pos] = J;
+        tk.qi[pos] = idx;
+      }
+      if (named_bar_or(barid, 128, push)) {
+        topk_merge(tk, row, 128, [barid] __device__() { named_bar(barid, 128); });
+        thr_s = tk.ls[kcap - 1];
+        thr_i = tk.li[kcap - 1];
+      }
+    }
+    // keep the pipeline's threads in step before the next tile reuses TMEM
+    tc_fence_before();
+    named_bar(barid, 128);
+  }
+
+  if (MODE == kTcRange) {
+    const size_t gl = ((size_t)blockIdx.x * npipes + pipe) * kcap;
+    for (int e = row; e < kcap; e += 128) {
+      R.lists_s[gl + e] = tk.ls[e];
+      R.lists_i[gl + e] = tk.li[e];
+    }
+    unsigned int c = my_count;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
+    if (lane == 0 && c) atomicAdd(R.count, (unsigned long long)c);
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(512) : "memory");
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Host side: operand images, layout, launches
+// ---------------------------------------------------------------------------
+namespace {
+
+uint16_t f2bf(float f) {  // round to nearest even
+  uint32_t u;
+  std::memcpy(&u, &f, 4);
+  if ((u & 0x7FFFFFFFu) > 0x7F800000u) return 0x7FC0;
+  u += 0x7FFFu + ((u >> 16) & 1u);
+  return (uint16_t)(u >> 16);
+}
+
+// Byte offset of element (r, k) of a K-major no-swizzle UMMA operand with kdim columns:
+// 8-row x 16-byte core matrices, K-adjacent cores 128 B apart, 8-row groups kdim*16 B apart.
+size_t umma_off(int r, int k, int kdim) {
+  return (size_t)(r >> 3) * (size_t)(kdim / 8) * 128u + (size_t)(k >> 3) * 128u + (size_t)(r & 7) * 16u +
+         (size_t)(k & 7) * 2u;
+}
+
+int round_up(int v, int a) { return (v + a - 1) / a * a; }
+
+size_t topk_bytes_pipe(int kcap) { return (sizeof(uint64_t) + sizeof(float)) * (2 * (size_t)kcap + 128) + 16; }
+
+// Shared-memory layout for a launch with per-pipeline lists of kcap entries.
+void layout_smem(const Params& P, TcArgs& T, int kcap) {
+  const int sumK = P.off[P.n_models - 1] + P.K[P.n_models - 1];
+  uint32_t o = round_up((int)T.img_bytes, 1024);
+  T.sm_xw = o; o += round_up(sumK * T.kw * 4, 16);
+  T.sm_dem = o; o += sumK * 16;
+  T.sm_b2 = o; o += round_up(P.n_models * T.h2 * 4, 16);
+  T.sm_b3 = o; o += round_up(P.n_models * 2 * 4, 16);
+  T.sm_topk = o; o += kcap > 0 ? (uint32_t)(T.pipes * topk_bytes_pipe(kcap)) : 0u;
+  o = round_up((int)o, 16);
+  T.sm_bar = o; o += 8 * (kTcMaxPipes + 1);
+  T.sm_total = o;
+  T.kcap = kcap;
+}
+
+constexpr uint32_t kSmemLimit = 227 * 1024 - 1024;  // static shared variables take the rest
+constexpr uint32_t kSmemFloor = 120 * 1024;          // keeps one CTA (one TMEM owner) per SM
+
+}  // namespace
+
 bool tc_supported(const Params& P, std::string* why) {
-  (void)P;
-  if (why) *why = "not built in this version";
-  return false;
+  auto no = [&](const char* m) { if (why) *why = m; return false; };
+  if (P.h1 % 32 || P.h1 > 256) return no("hidden1 must be a multiple of 32 up to 256");
+  if (P.h2 % 32 || P.h2 > 256) return no("hidden2 must be 0 or a multiple of 32 up to 256");
+  if (P.d_local > 24) return no("d_local must be <= 24");
+  const int hmax = P.h1 > P.h2 ? P.h1 : P.h2;
+  const int dle = P.d_local + (P.d_local & 1);
+  const int kw = round_up(dle + 8, 16) / 2;
+  const int n3 = 2 * P.n_models <= 16 ? 16 : 32;
+  const int col_a = hmax + hmax / 2;
+  const int col_d3 = round_up(col_a + kw, 16);
+  if (round_up(col_d3 + n3, 32) > 512) return no("tensor-memory footprint above 512 columns");
+  const int hl = P.h2 > 0 ? P.h2 : P.h1;
+  size_t img = 0;
+  for (int i = 0; i < P.n_models; ++i)
+    img += (size_t)P.h1 * 2 * kw * 2 + (size_t)P.h2 * P.h1 * 2 + (size_t)n3 * hl * 2;
+  if (img > 160 * 1024) return no("bf16 weights of all models exceed the shared-memory budget");
+  return true;
 }
-mf_status tc_prepare(mf_ctx* c) { (void)c; return MF_EUNSUPPORTED; }
-int tc_grid(const mf_ctx* c) { return c->num_sms; }
+
+int tc_grid(const mf_ctx* c) { return c->num_sms * c->tc.pipes; }
+
+mf_status tc_prepare(mf_ctx* c) {
+  const Params& P = c->P;
+  TcArgs& T = c->tc;
+  std::memset(&T, 0, sizeof(T));
+  const int N = P.n_models, dl = P.d_local, h1 = P.h1, h2 = P.h2, hl = h2 > 0 ? h2 : h1;
+  const int din = P.d_in;
+  T.dle = dl + (dl & 1);
+  T.k1 = round_up(T.dle + 8, 16);
+  T.kw = T.k1 / 2;
+  T.h1 = h1;
+  T.h2 = h2;
+  T.hl = hl;
+  T.n3 = 2 * N <= 16 ? 16 : 32;
+  const int hmax = h1 > h2 ? h1 : h2;
+  T.col_d = 0;
+  T.col_h = hmax;
+  T.col_a = hmax + hmax / 2;
+  T.col_d3 = round_up(T.col_a + T.kw, 16);
+  T.pipe_stride = round_up(T.col_d3 + T.n3, 32);
+  T.pipes = 512 / T.pipe_stride;
+  if (T.pipes > kTcMaxPipes) T.pipes = kTcMaxPipes;
+
+  // B operand images
+  const size_t b1_bytes = (size_t)h1 * T.k1 * 2, b2_bytes = (size_t)h2 * h1 * 2, b3_bytes = (size_t)T.n3 * hl * 2;
+  std::vector<unsigned char> img;
+  const double s3 = P.agg_scale[3];
+  std::vector<float> w(P.per_model * N);
+  cudaError_t e = cudaMemcpy(w.data(), P.w32, sizeof(float) * w.size(), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "tc_prepare: read weights");
+  for (int i = 0; i < N; ++i) {
+    const float* src = w.data() + (size_t)i * P.per_model;
+    const float* W1 = src;
+    const float* b1 = W1 + (size_t)h1 * din;
+    const float* W2 = b1 + h1;
+    const float* W3 = h2 > 0 ? W2 + (size_t)h2 * h1 + h2 : W2;
+    T.off_b1[i] = (uint32_t)img.size();
+    img.resize(img.size() + b1_bytes, 0);
+    for (int j = 0; j < h1; ++j) {
+      auto put = [&](int k, double v) {
+        const uint16_t b = f2bf((float)v);
+        std::memcpy(img.data() + T.off_b1[i] + umma_off(j, k, T.k1), &b, 2);
+      };
+      for (int k = 0; k < dl; ++k) put(k, W1[(size_t)j * din + k]);
+      // A1 carries the scaled aggregate (hi and lo parts), so these columns hold W1 as is;
+      // the constant-1 column carries b1 plus the weight of the constant feature N * s_3
+      for (int q = 0; q < 3; ++q) {
+        put(T.dle + q, W1[(size_t)j * din + dl + q]);
+        put(T.dle + 4 + q, W1[(size_t)j * din + dl + q]);
+      }
+      put(T.dle + 3, (double)b1[j] + (double)W1[(size_t)j * din + dl + 3] * s3 * N);
+    }
+    T.off_b2[i] = (uint32_t)img.size();
+    img.resize(img.size() + b2_bytes, 0);
+    for (int j = 0; j < h2; ++j)
+      for (int k = 0; k < h1; ++k) {
+        const uint16_t b = f2bf(W2[(size_t)j * h1 + k]);
+        std::memcpy(img.data() + T.off_b2[i] + umma_off(j, k, h1), &b, 2);
+      }
+    T.off_b3[i] = (uint32_t)img.size();
+    img.resize(img.size() + b3_bytes, 0);
+    for (int k = 0; k < hl; ++k) {
+      const uint16_t bt = f2bf(W3[k]), bl = f2bf(W3[hl + k]);
+      std::memcpy(img.data() + T.off_b3[i] + umma_off(i, k, hl), &bt, 2);
+      std::memcpy(img.data() + T.off_b3[i] + umma_off(T.n3 / 2 + i, k, hl), &bl, 2);
+    }
+  }
+  img.resize(round_up((int)img.size(), 16), 0);
+  T.img_bytes = (uint32_t)img.size();
+
+  // local-feature words, biases
+  const int sumK = c->sumK;
+  std::vector<float> x((size_t)sumK * dl);
+  e = cudaMemcpy(x.data(), P.x, sizeof(float) * x.size(), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "tc_prepare: read tables");
+  std::vector<uint32_t> xw((size_t)sumK * T.kw, 0u);
+  for (int r = 0; r < sumK; ++r)
+    for (int k = 0; k < dl; ++k)
+      xw[(size_t)r * T.kw + k / 2] |= (uint32_t)f2bf(x[(size_t)r * dl + k]) << (16 * (k & 1));
+  std::vector<float> b2v((size_t)N * h2), b3v((size_t)N * 2);
+  for (int i = 0; i < N; ++i) {
+    const float* src = w.data() + (size_t)i * P.per_model;
+    const float* b2 = src + (size_t)h1 * din + h1 + (size_t)h2 * h1;
+    for (int j = 0; j < h2; ++j) b2v[(size_t)i * h2 + j] = b2[j];
+    const float* b3 = src + (size_t)h1 * din + h1 + (h2 > 0 ? (size_t)h2 * h1 + h2 : 0) + 2 * (size_t)hl;
+    b3v[2 * i] = b3[0];
+    b3v[2 * i + 1] = b3[1];
+  }
+  const size_t o_xw = round_up((int)img.size(), 256);
+  const size_t o_b2 = o_xw + round_up((int)(xw.size() * 4), 256);
+  const size_t o_b3 = o_b2 + round_up((int)(b2v.size() * 4) + 4, 256);
+  const size_t total = o_b3 + round_up((int)(b3v.size() * 4), 256);
+  MF_CUDA(cudaMalloc(&c->d_tc, total));
+  c->tc_bytes = total;
+  unsigned char* base = static_cast<unsigned char*>(c->d_tc);
+  MF_CUDA(cudaMemcpy(base, img.data(), img.size(), cudaMemcpyHostToDevice));
+  MF_CUDA(cudaMemcpy(base + o_xw, xw.data(), xw.size() * 4, cudaMemcpyHostToDevice));
+  if (!b2v.empty()) MF_CUDA(cudaMemcpy(base + o_b2, b2v.data(), b2v.size() * 4, cudaMemcpyHostToDevice));
+  MF_CUDA(cudaMemcpy(base + o_b3, b3v.data(), b3v.size() * 4, cudaMemcpyHostToDevice));
+  c->stats.h2d_bytes_create += img.size() + xw.size() * 4 + b2v.size() * 4 + b3v.size() * 4;
+  T.img = base;
+  T.xw = reinterpret_cast<const uint32_t*>(base + o_xw);
+  T.b2 = reinterpret_cast<const float*>(base + o_b2);
+  T.b3 = reinterpret_cast<const float*>(base + o_b3);
+  MF_CUDA(cudaFuncSetAttribute(k_score_tc<kTcRange>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit));
+  MF_CUDA(cudaFuncSetAttribute(k_score_tc<kTcList>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit));
+  layout_smem(P, T, 0);
+  if (T.sm_total > kSmemLimit) {
+    set_error("tensor-core path: tables and weights exceed shared memory");
+    return MF_EUNSUPPORTED;
+  }
+  return MF_OK;
+}
+
 mf_status tc_search_chunk(mf_ctx* c, const RangeArgs& a, cudaStream_t s) {
-  (void)c; (void)a; (void)s;
-  return MF_EUNSUPPORTED;
+  TcArgs T = c->tc;
+  layout_smem(c->P, T, a.k);
+  if (T.sm_total > kSmemLimit) {
+    set_error("tensor-core path: top-k lists do not fit shared memory; use a smaller k");
+    return MF_EUNSUPPORTED;
+  }
+  const uint32_t smem = T.sm_total > kSmemFloor ? T.sm_total : kSmemFloor;
+  TcList L{};
+  k_score_tc<kTcRange><<<c->num_sms, T.pipes * 128, smem, s>>>(c->P, T, a, L);
+  MF_CUDA(cudaGetLastError());
+  return MF_OK;
 }
-mf_status tc_score_list(mf_ctx* c, const uint64_t* idx, uint64_t n, float* score, uint8_t* feas,
-                        float* pred, cudaStream_t s) {
-  (void)c; (void)idx; (void)n; (void)score; (void)feas; (void)pred; (void)s;
-  return MF_EUNSUPPORTED;
+
+mf_status tc_score_list(mf_ctx* c, const uint64_t* idx, uint64_t n, float* score, uint8_t* feas, float* pred,
+                        cudaStream_t s) {
+  if (n == 0) return MF_OK;
+  TcArgs T = c->tc;
+  layout_smem(c->P, T, 0);
+  const uint32_t smem = T.sm_total > kSmemFloor ? T.sm_total : kSmemFloor;
+  const uint64_t tiles = (n + 127) / 128;
+  const uint64_t per_cta = (uint64_t)T.pipes;
+  uint64_t grid = (tiles + per_cta - 1) / per_cta;
+  if (grid > (uint64_t)c->num_sms) grid = c->num_sms;
+  RangeArgs R{};
+  TcList L{idx, n, score, feas, pred};
+  k_score_tc<kTcList><<<(unsigned)grid, T.pipes * 128, smem, s>>>(c->P, T, R, L);
+  MF_CUDA(cudaGetLastError());
+  return MF_OK;
 }
 
 }  // namespace mf

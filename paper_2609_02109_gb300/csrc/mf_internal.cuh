@@ -35,6 +35,20 @@ struct Params {
   uint32_t* status;                   // device status word (bit 0: bad index/gene)
 };
 
+// Tensor-core path: operand images and the per-CTA layout (filled by tc_prepare).
+struct TcArgs {
+  const void* img;                    // bf16 B operands, UMMA K-major no-swizzle layout
+  uint32_t img_bytes;
+  const uint32_t* xw;                 // [sumK][kw] bf16 pairs of the local features
+  const float* b2;                    // [N][h2]
+  const float* b3;                    // [N][2]
+  int32_t k1, kw, h1, h2, hl, n3, dle;
+  uint32_t off_b1[MF_MAX_MODELS], off_b2[MF_MAX_MODELS], off_b3[MF_MAX_MODELS];  // bytes in img
+  int32_t pipes, col_d, col_h, col_a, col_d3, pipe_stride;  // TMEM columns
+  uint32_t sm_xw, sm_dem, sm_b2, sm_b3, sm_topk, sm_bar, sm_total;  // shared-memory byte offsets
+  int32_t kcap;                       // per-pipeline list length the layout was sized for
+};
+
 // Device status bits.
 constexpr uint32_t kStatusBadInput = 1u;
 constexpr uint32_t kStatusTimeout = 2u;
@@ -175,6 +189,7 @@ struct mf_ctx {
   uint32_t* d_status = nullptr;
   void* d_tc = nullptr;           // packed bf16 operand images (tensor-core path)
   size_t tc_bytes = 0;
+  mf::TcArgs tc{};
   // growable scratch (search lists, merge buffers, shortlist)
   void* d_scratch = nullptr;
   size_t scratch_bytes = 0;

@@ -41,9 +41,14 @@ def near_threshold(prob, ref_pred, ref_agg, prec="fp32"):
 
 
 def check_scores(prob, got_score, got_feas, ref_score, ref_feas, ref_pred, ref_agg, prec="fp32",
-                 got_pred=None):
+                 got_pred=None, pred_scale=None):
     """Element-wise parity of a score batch.  Returns the number of near-threshold
-    candidates excluded from the exact feasibility comparison."""
+    candidates excluded from the exact feasibility comparison.
+
+    Per-model outputs: fp32 within 1e-5 of max(|y|, RMS of the head over the batch);
+    bf16 within 2e-2 of max(|y|, c), c = the oracle's condition scale of the head,
+    |b3| + sum_k |W3_k| |h_k| (bf16 rounding errors scale with the magnitude of the
+    terms of the final dot product, which can cancel to a much smaller |y|)."""
     got_score = np.asarray(got_score, dtype=np.float64)
     got_feas = np.asarray(got_feas).astype(bool)
     near = near_threshold(prob, ref_pred, ref_agg, prec)
@@ -58,8 +63,12 @@ def check_scores(prob, got_score, got_feas, ref_score, ref_feas, ref_pred, ref_a
     if got_pred is not None:
         gp = np.asarray(got_pred, dtype=np.float64)
         for h in range(2):
-            rms = np.sqrt(np.mean(ref_pred[..., h] ** 2, axis=0, keepdims=True))
-            d = np.abs(gp[..., h] - ref_pred[..., h]) / np.maximum(np.abs(ref_pred[..., h]), rms)
+            if pred_scale is not None:
+                den = np.maximum(np.abs(ref_pred[..., h]), pred_scale[..., h])
+            else:
+                rms = np.sqrt(np.mean(ref_pred[..., h] ** 2, axis=0, keepdims=True))
+                den = np.maximum(np.abs(ref_pred[..., h]), rms)
+            d = np.abs(gp[..., h] - ref_pred[..., h]) / np.maximum(den, 1e-30)
             assert d.max() <= RTOL[prec], f"head {h} error {d.max():.3g}"
     return int(near.sum())
 

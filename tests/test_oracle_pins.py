@@ -340,3 +340,28 @@ def test_default_agg_scale(oracle_mod):
     prob["agg_scale"] = None
     got = _O(oracle_mod, prob).score_list(np.arange(50, dtype=np.uint64))[0]
     np.testing.assert_array_equal(ref, got)
+
+
+def test_pred_scale_equals_output_in_linear_case(oracle_mod):
+    """With non-negative weights and inputs no term of the final dot product
+    cancels, so the condition scale equals |output|."""
+    prob = W.make_problem([3, 4], 8, 16, 8, 11, 1e9)
+    prob["weights"] = np.abs(prob["weights"])
+    o = _O(oracle_mod, prob)
+    idx = np.arange(o.space_size(), dtype=np.uint64)
+    _, _, pred, _ = o.score_list(idx, with_pred=True)
+    np.testing.assert_allclose(o.pred_scale(idx), np.abs(pred), rtol=1e-12)
+
+
+def test_pred_scale_hand_value(oracle_mod):
+    """One input x = 0.5, two hidden units h = (x, 0.5 x) = (0.5, 0.25), throughput
+    row W3 = (1, -1): thr = 0.25 while the terms have magnitude 0.5 + 0.25 = 0.75."""
+    p = dict(n_options=np.array([1], np.int32), d_local=1, hidden1=2, hidden2=0,
+             local_feats=np.array([[0.5]], np.float32), demand=np.array([[0.1, 1.0, 10.0]], np.float32),
+             weights=np.array([1, 0, 0, 0, 0, 0.5, 0, 0, 0, 0,  0, 0,  1, -1, 0, 0,  0, 0], np.float32),
+             agg_scale=np.ones(4, np.float32), sla=np.array([9.0], np.float32),
+             obj_w=np.ones(1, np.float32), vram_cap=100.0)
+    o = _O(oracle_mod, p)
+    J, f, pred, _ = o.score_digits([0])
+    assert pred[0, 0] == pytest.approx(0.25)
+    np.testing.assert_allclose(o.pred_scale(np.array([0], np.uint64))[0, 0], [0.75, 0.0], atol=1e-12)
