@@ -20,10 +20,16 @@
 // that the pipeline's threads wait on (bounded; a wait that gives up raises the
 // status word and the kernel runs to completion without further waits).
 //
-// Biases: b1 rides in A1's constant-1 column, b2 is added in the layer-2
-// epilogue, b3 in the final epilogue.  The aggregate enters layer 1 as a bf16
-// hi/lo pair (two columns per component with the same weight), so its rounding
-// error is ~2^-16 rather than 2^-9.
+// Biases ride in the MMAs: b1 in A1's constant-1 column; b2 and b3 through a
+// constant block of ones that sits in tensor memory right after each layer's
+// activations (one extra K = 16 step whose B rows hold the bias as a bf16 hi/lo
+// pair), so the epilogues are only load -> ReLU + round -> store.  The
+// aggregate enters layer 1 as a bf16 hi/lo pair as well (two columns per
+// component with the same weight), so its rounding error is ~2^-16, not 2^-9.
+//
+// Each thread keeps its candidate's option rows in shared memory and steps them
+// from tile to tile by adding the digits of the tile stride with carries, so no
+// division runs in the hot loop.
 #include <cuda_bf16.h>
 
 #include <cstring>
@@ -171,13 +177,13 @@ struct TcList {
 struct PipeWait {
   volatile int* abort;
   uint32_t* status;
-  // Bounded wait for `parity` of `bar`; on giving up flags the status word and
-  // makes every later wait return at once.
+  // Bounded wait for `parity` of `bar`; on giving up it flags the status word and
+  // every later wait returns at once, so the kernel still runs to its end.
   __device__ __forceinline__ void operator()(uint64_t* bar, uint32_t parity) const {
+    if (*abort) return;
     uint32_t n = 0;
-    while (!*abort) {
-      if (mbar_try_wait(bar, parity)) return;
-      if (++n > kWaitLimit) {
+    while (!mbar_try_wait(bar, parity)) {
+      if (++n == kWaitLimit) {
         *abort = 1;
         atomicOr(status, kStatusTimeout);
         return;
@@ -200,10 +206,11 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   const int npipes = T.pipes;
 
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + T.sm_bar);
-  uint32_t* xw_s = reinterpret_cast<uint32_t*>(smem + T.sm_xw);
+  const uint4* xw_s = reinterpret_cast<const uint4*>(smem + T.sm_xw);
   float4* dem_s = reinterpret_cast<float4*>(smem + T.sm_dem);
-  float* b2_s = reinterpret_cast<float*>(smem + T.sm_b2);
-  float* b3_s = reinterpret_cast<float*>(smem + T.sm_b3);
+  uint64_t* desc_s = reinterpret_cast<uint64_t*>(smem + T.sm_desc);
+  // this thread's current option row of every model: rows[i * 128 + row]
+  uint16_t* rows = reinterpret_cast<uint16_t*>(smem + T.sm_rows) + (size_t)pipe * MF_MAX_MODELS * 128;
 
   if (tid == 0) {
     s_abort = 0;
@@ -217,6 +224,7 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
   __syncthreads();
+  const uint32_t smem_base = smem_u32(smem);
   if (tid == 0) {
     // weights: one TMA bulk copy per 32 KB piece, all completing on bars[0]
     mbar_arrive_expect_tx(&bars[0], T.img_bytes);
@@ -225,12 +233,19 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
       bulk_g2s(smem + o, static_cast<const unsigned char*>(T.img) + o, b, &bars[0]);
     }
   }
-  // option tables and biases with ordinary loads
+  // UMMA descriptors of every model's three B operands
+  if (tid < N) {
+    desc_s[3 * tid + 0] = smem_desc(smem_base + T.off_b1[tid], 128u, (uint32_t)(T.k1 / 8) * 128u);
+    desc_s[3 * tid + 1] = smem_desc(smem_base + T.off_b2[tid], 128u, (uint32_t)((T.h1 + 16) / 8) * 128u);
+    desc_s[3 * tid + 2] = smem_desc(smem_base + T.off_b3[tid], 128u, (uint32_t)((T.hl + 16) / 8) * 128u);
+  }
+  // option tables with ordinary loads
   const int sumK = P.off[N - 1] + P.K[N - 1];
-  for (int e = tid; e < sumK * T.kw; e += blockDim.x) xw_s[e] = T.xw[e];
+  {
+    uint32_t* xw32 = reinterpret_cast<uint32_t*>(smem + T.sm_xw);
+    for (int e = tid; e < sumK * T.kw; e += blockDim.x) xw32[e] = T.xw[e];
+  }
   for (int e = tid; e < sumK; e += blockDim.x) dem_s[e] = P.dem[e];
-  for (int e = tid; e < N * T.h2; e += blockDim.x) b2_s[e] = T.b2[e];
-  for (int e = tid; e < 2 * N; e += blockDim.x) b3_s[e] = T.b3[e];
 
   // per-pipeline running top-k (range mode)
   CtaTopK tk{};
@@ -258,25 +273,30 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   tc_fence_after();
   const uint32_t tmem = s_tmem;
   const PipeWait wait_bar{&s_abort, P.status};
-  wait_bar(&bars[0], 0);  // weights landed
 
   const uint32_t tp = tmem + (uint32_t)(pipe * T.pipe_stride);
   const uint32_t lane_off = (uint32_t)(wq * 32) << 16;
-  const uint32_t tD = tp + T.col_d, tH = tp + T.col_h, tA = tp + T.col_a, tD3 = tp + T.col_d3;
+  const uint32_t tD = tp + T.col_d, tA = tp + T.col_a, tD3 = tp + T.col_d3, tOnes = tp + T.col_ones;
+  const uint32_t tH1 = tOnes - (uint32_t)(T.h1 / 2);                        // layer-2 A operand
+  const uint32_t tH2 = T.h2 > 0 ? tOnes - (uint32_t)(T.h2 / 2) : tH1;       // layer-3 A operand
   const bool leader = (wq == 0 && lane == 0);
   uint64_t* mbar = &bars[1 + pipe];
   uint32_t phase = 0;
   const int barid = 1 + pipe;
-  const uint32_t smem_base = smem_u32(smem);
   const uint32_t id1 = idesc_bf16(T.h1), id2 = idesc_bf16(T.h2), id3 = idesc_bf16(T.n3);
-  const uint32_t sbo1 = (uint32_t)(T.k1 / 8) * 128u, sbo2 = (uint32_t)(T.h1 / 8) * 128u,
-                 sbo3 = (uint32_t)(T.hl / 8) * 128u;
+  const int s1 = T.k1 / 16, s2 = T.h1 / 16 + 1, s3 = T.hl / 16 + 1;
   const float vcap = P.vram_cap;
+
+  {  // constant ones block: word 0 = (1, 1) feeds the bias hi/lo rows of B2 and B3
+    uint32_t v[8] = {0x3F803F80u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
+    tmem_st_x8(tOnes + lane_off, v);
+    tmem_wait_st();
+  }
+  wait_bar(&bars[0], 0);  // weights landed
 
   float thr_s = -INFINITY;
   uint64_t thr_i = kEmptyIdx;
   if (MODE == kTcRange) {
-    named_bar(barid, 128);
     thr_s = tk.ls[kcap - 1];
     thr_i = tk.li[kcap - 1];
   }
@@ -286,52 +306,67 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   const uint64_t gpipe = (uint64_t)blockIdx.x * npipes + pipe;
   const uint64_t gstride = (uint64_t)gridDim.x * npipes;
 
+  // range mode: digits of the first candidate, then stepped per tile
+  if (MODE == kTcRange && gpipe * 128 < n) {
+    const uint64_t idx0 = R.base + gpipe * 128 + row;
+    for (int i = 0; i < N; ++i) rows[i * 128 + row] = (uint16_t)(P.off[i] + (int)((idx0 / P.stride[i]) % P.K[i]));
+  }
+
   auto issue_mma1 = [&](int i) {
-    const uint32_t b = smem_base + T.off_b1[i];
-    for (int s = 0; s < T.k1 / 16; ++s)
-      mma_ts(tD, tA + 8 * s, smem_desc(b + 256u * s, 128u, sbo1), id1, s > 0);
+    const uint64_t d = desc_s[3 * i + 0];
+    for (int s = 0; s < s1; ++s) mma_ts(tD, tA + 8 * s, d + 16u * s, id1, s > 0);
   };
   auto issue_mma2 = [&](int i) {
-    const uint32_t b = smem_base + T.off_b2[i];
-    for (int s = 0; s < T.h1 / 16; ++s)
-      mma_ts(tD, tH + 8 * s, smem_desc(b + 256u * s, 128u, sbo2), id2, s > 0);
+    const uint64_t d = desc_s[3 * i + 1];
+    for (int s = 0; s < s2; ++s) mma_ts(tD, tH1 + 8 * s, d + 16u * s, id2, s > 0);
   };
   auto issue_mma3 = [&](int i) {
-    const uint32_t b = smem_base + T.off_b3[i];
-    for (int s = 0; s < T.hl / 16; ++s)
-      mma_ts(tD3, tH + 8 * s, smem_desc(b + 256u * s, 128u, sbo3), id3, (i > 0 || s > 0));
+    const uint64_t d = desc_s[3 * i + 2];
+    for (int s = 0; s < s3; ++s) mma_ts(tD3, tH2 + 8 * s, d + 16u * s, id3, (i > 0 || s > 0));
   };
-  // fp32 accumulators [cols c0, c0+32) -> (+ bias) -> ReLU -> bf16 pairs at H[c0/2 ..)
-  auto epilogue = [&](int width, const float* bias) {
+  // fp32 accumulators [0, width) -> ReLU -> bf16 pairs at dst
+  auto epilogue = [&](int width, uint32_t dst) {
     for (int c0 = 0; c0 < width; c0 += 32) {
       uint32_t r[32];
       tmem_ld_x32(tD + lane_off + c0, r);
       tmem_wait_ld();
-      if (bias) {
-#pragma unroll
-        for (int j = 0; j < 32; ++j) r[j] = __float_as_uint(__uint_as_float(r[j]) + bias[c0 + j]);
-      }
       uint32_t h[16];
 #pragma unroll
       for (int j = 0; j < 16; ++j) h[j] = relu_bf16x2(r[2 * j], r[2 * j + 1]);
-      tmem_st_x16(tH + lane_off + (c0 >> 1), h);
+      tmem_st_x16(dst + lane_off + (c0 >> 1), h);
     }
   };
 
+  bool first_tile = true;
   for (uint64_t tile = gpipe; tile * 128 < n; tile += gstride) {
     const uint64_t t = tile * 128 + row;
     bool valid = t < n;
     uint64_t idx = 0;
-    if (valid) idx = MODE == kTcRange ? R.base + t : L.idx[t];
-    if (MODE == kTcList && valid && idx >= P.total) {
-      atomicOr(P.status, kStatusBadInput);
-      valid = false;
+    if (MODE == kTcRange) {
+      idx = R.base + t;
+      if (!first_tile) {  // add the tile stride to the digits, last model first
+        uint32_t carry = 0;
+        for (int i = N - 1; i >= 0; --i) {
+          uint32_t d = (uint32_t)rows[i * 128 + row] - (uint32_t)P.off[i] + T.step[i] + carry;
+          carry = d >= (uint32_t)P.K[i];
+          if (carry) d -= (uint32_t)P.K[i];
+          rows[i * 128 + row] = (uint16_t)(P.off[i] + (int)d);
+        }
+      }
+    } else {
+      if (valid) idx = L.idx[t];
+      if (valid && idx >= P.total) {
+        atomicOr(P.status, kStatusBadInput);
+        valid = false;
+      }
+      if (!valid) idx = 0;  // compute on candidate 0, discard at the end
+      for (int i = 0; i < N; ++i) rows[i * 128 + row] = (uint16_t)(P.off[i] + digit_of(P, idx, i));
     }
-    if (!valid) idx = 0;  // compute on candidate 0, discard at the end
+    first_tile = false;
     // aggregate state (fp32, model order) and its bf16 hi/lo words
     float A0 = 0.f, A1 = 0.f, A2 = 0.f;
     for (int i = 0; i < N; ++i) {
-      const float4 d = dem_s[P.off[i] + digit_of(P, idx, i)];
+      const float4 d = dem_s[rows[i * 128 + row]];
       A0 += d.x; A1 += d.y; A2 += d.z;
     }
     uint32_t aw[4];
@@ -348,21 +383,23 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     }
     const int awo = T.dle >> 1;
     auto write_a1 = [&](int i) {
-      const int r0 = (P.off[i] + digit_of(P, idx, i)) * T.kw;
+      const uint4* src = xw_s + (size_t)rows[i * 128 + row] * (T.kw >> 2);
       // word j: local-feature pair, or aggregate word j - awo for awo <= j < awo + 4
-      auto word = [&](int j) -> uint32_t {
+      auto pick = [&](int j, uint32_t x) -> uint32_t {
         const int a = j - awo;
-        return a == 0 ? aw[0] : a == 1 ? aw[1] : a == 2 ? aw[2] : a == 3 ? aw[3] : xw_s[r0 + j];
+        return a == 0 ? aw[0] : a == 1 ? aw[1] : a == 2 ? aw[2] : a == 3 ? aw[3] : x;
       };
       if (T.kw == 8) {
-        uint32_t v[8];
-#pragma unroll
-        for (int j = 0; j < 8; ++j) v[j] = word(j);
+        const uint4 q0 = src[0], q1 = src[1];
+        uint32_t v[8] = {pick(0, q0.x), pick(1, q0.y), pick(2, q0.z), pick(3, q0.w),
+                         pick(4, q1.x), pick(5, q1.y), pick(6, q1.z), pick(7, q1.w)};
         tmem_st_x8(tA + lane_off, v);
       } else {
-        uint32_t v[16];
-#pragma unroll
-        for (int j = 0; j < 16; ++j) v[j] = word(j);
+        const uint4 q0 = src[0], q1 = src[1], q2 = src[2], q3 = src[3];
+        uint32_t v[16] = {pick(0, q0.x),  pick(1, q0.y),  pick(2, q0.z),  pick(3, q0.w),
+                          pick(4, q1.x),  pick(5, q1.y),  pick(6, q1.z),  pick(7, q1.w),
+                          pick(8, q2.x),  pick(9, q2.y),  pick(10, q2.z), pick(11, q2.w),
+                          pick(12, q3.x), pick(13, q3.y), pick(14, q3.z), pick(15, q3.w)};
         tmem_st_x16(tA + lane_off, v);
       }
     };
@@ -381,7 +418,7 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
       wait_bar(mbar, phase);
       phase ^= 1u;
       tc_fence_after();
-      epilogue(T.h1, nullptr);  // layer 1 (bias in the constant column)
+      epilogue(T.h1, tH1);  // layer 1 (bias in the constant column)
       if (T.h2 > 0) {
         tmem_wait_st();
         tc_fence_before();
@@ -394,7 +431,7 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
         wait_bar(mbar, phase);
         phase ^= 1u;
         tc_fence_after();
-        epilogue(T.h2, b2_s + i * T.h2);  // layer 2
+        epilogue(T.h2, tH2);  // layer 2 (bias through the ones block)
       }
       if (i + 1 < N) write_a1(i + 1);
       tmem_wait_st();
@@ -428,10 +465,8 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
       if (i >= N) break;
-      const float dthr = __uint_as_float(d3[i]);
-      const float dlat = __uint_as_float(half3 == 8 ? d3[(8 + i) & 31] : d3[(16 + i) & 31]);
-      const float thr = out_act(P, dthr + b3_s[2 * i]);
-      const float lat = out_act(P, dlat + b3_s[2 * i + 1]);
+      const float thr = out_act(P, __uint_as_float(d3[i]));
+      const float lat = out_act(P, __uint_as_float(half3 == 8 ? d3[(8 + i) & 31] : d3[(16 + i) & 31]));
       if (MODE == kTcList && valid && L.pred) {
         L.pred[(t * N + i) * 2 + 0] = thr;
         L.pred[(t * N + i) * 2 + 1] = lat;
@@ -472,9 +507,6 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
         thr_i = tk.li[kcap - 1];
       }
     }
-    // keep the pipeline's threads in step before the next tile reuses TMEM
-    tc_fence_before();
-    named_bar(barid, 128);
   }
 
   if (MODE == kTcRange) {
@@ -509,6 +541,13 @@ uint16_t f2bf(float f) {  // round to nearest even
   return (uint16_t)(u >> 16);
 }
 
+float bf2f(uint16_t b) {
+  const uint32_t u = (uint32_t)b << 16;
+  float f;
+  std::memcpy(&f, &u, 4);
+  return f;
+}
+
 // Byte offset of element (r, k) of a K-major no-swizzle UMMA operand with kdim columns:
 // 8-row x 16-byte core matrices, K-adjacent cores 128 B apart, 8-row groups kdim*16 B apart.
 size_t umma_off(int r, int k, int kdim) {
@@ -520,14 +559,20 @@ int round_up(int v, int a) { return (v + a - 1) / a * a; }
 
 size_t topk_bytes_pipe(int kcap) { return (sizeof(uint64_t) + sizeof(float)) * (2 * (size_t)kcap + 128) + 16; }
 
+size_t image_bytes(const Params& P, int k1, int n3) {
+  const int hl = P.h2 > 0 ? P.h2 : P.h1;
+  const size_t per = (size_t)P.h1 * k1 * 2 + (size_t)P.h2 * (P.h1 + 16) * 2 + (size_t)n3 * (hl + 16) * 2;
+  return per * P.n_models;
+}
+
 // Shared-memory layout for a launch with per-pipeline lists of kcap entries.
 void layout_smem(const Params& P, TcArgs& T, int kcap) {
   const int sumK = P.off[P.n_models - 1] + P.K[P.n_models - 1];
   uint32_t o = round_up((int)T.img_bytes, 1024);
   T.sm_xw = o; o += round_up(sumK * T.kw * 4, 16);
   T.sm_dem = o; o += sumK * 16;
-  T.sm_b2 = o; o += round_up(P.n_models * T.h2 * 4, 16);
-  T.sm_b3 = o; o += round_up(P.n_models * 2 * 4, 16);
+  T.sm_rows = o; o += T.pipes * MF_MAX_MODELS * 128 * 2;
+  T.sm_desc = o; o += 8 * 3 * MF_MAX_MODELS;
   T.sm_topk = o; o += kcap > 0 ? (uint32_t)(T.pipes * topk_bytes_pipe(kcap)) : 0u;
   o = round_up((int)o, 16);
   T.sm_bar = o; o += 8 * (kTcMaxPipes + 1);
@@ -547,16 +592,12 @@ bool tc_supported(const Params& P, std::string* why) {
   if (P.d_local > 24) return no("d_local must be <= 24");
   const int hmax = P.h1 > P.h2 ? P.h1 : P.h2;
   const int dle = P.d_local + (P.d_local & 1);
-  const int kw = round_up(dle + 8, 16) / 2;
+  const int k1 = round_up(dle + 8, 16);
   const int n3 = 2 * P.n_models <= 16 ? 16 : 32;
-  const int col_a = hmax + hmax / 2;
-  const int col_d3 = round_up(col_a + kw, 16);
+  const int col_a = hmax + hmax / 2 + 8;
+  const int col_d3 = round_up(col_a + k1 / 2, 16);
   if (round_up(col_d3 + n3, 32) > 512) return no("tensor-memory footprint above 512 columns");
-  const int hl = P.h2 > 0 ? P.h2 : P.h1;
-  size_t img = 0;
-  for (int i = 0; i < P.n_models; ++i)
-    img += (size_t)P.h1 * 2 * kw * 2 + (size_t)P.h2 * P.h1 * 2 + (size_t)n3 * hl * 2;
-  if (img > 160 * 1024) return no("bf16 weights of all models exceed the shared-memory budget");
+  if (image_bytes(P, k1, n3) > 160 * 1024) return no("bf16 weights of all models exceed the shared-memory budget");
   return true;
 }
 
@@ -578,60 +619,70 @@ mf_status tc_prepare(mf_ctx* c) {
   const int hmax = h1 > h2 ? h1 : h2;
   T.col_d = 0;
   T.col_h = hmax;
-  T.col_a = hmax + hmax / 2;
+  T.col_ones = hmax + hmax / 2;
+  T.col_a = T.col_ones + 8;
   T.col_d3 = round_up(T.col_a + T.kw, 16);
   T.pipe_stride = round_up(T.col_d3 + T.n3, 32);
   T.pipes = 512 / T.pipe_stride;
   if (T.pipes > kTcMaxPipes) T.pipes = kTcMaxPipes;
 
-  // B operand images
-  const size_t b1_bytes = (size_t)h1 * T.k1 * 2, b2_bytes = (size_t)h2 * h1 * 2, b3_bytes = (size_t)T.n3 * hl * 2;
+  // B operand images (K-major): B1 [h1 x k1], B2 [h2 x (h1 + 16)], B3 [n3 x (hl + 16)]
+  const int k2 = h1 + 16, k3 = hl + 16;
+  const size_t b1_bytes = (size_t)h1 * T.k1 * 2, b2_bytes = (size_t)h2 * k2 * 2, b3_bytes = (size_t)T.n3 * k3 * 2;
   std::vector<unsigned char> img;
   const double s3 = P.agg_scale[3];
   std::vector<float> w(P.per_model * N);
   cudaError_t e = cudaMemcpy(w.data(), P.w32, sizeof(float) * w.size(), cudaMemcpyDeviceToHost);
   if (e != cudaSuccess) return cuda_fail(e, "tc_prepare: read weights");
+  auto put = [&](uint32_t base, int r, int k, int kdim, double v) {
+    const uint16_t b = f2bf((float)v);
+    std::memcpy(img.data() + base + umma_off(r, k, kdim), &b, 2);
+  };
+  // a bias as a bf16 pair (hi, lo) whose sum carries ~16 mantissa bits
+  auto put_bias = [&](uint32_t base, int r, int k, int kdim, float v) {
+    const uint16_t hi = f2bf(v);
+    put(base, r, k, kdim, bf2f(hi));
+    put(base, r, k + 1, kdim, (double)v - (double)bf2f(hi));
+  };
   for (int i = 0; i < N; ++i) {
     const float* src = w.data() + (size_t)i * P.per_model;
     const float* W1 = src;
     const float* b1 = W1 + (size_t)h1 * din;
     const float* W2 = b1 + h1;
-    const float* W3 = h2 > 0 ? W2 + (size_t)h2 * h1 + h2 : W2;
+    const float* b2 = W2 + (size_t)h2 * h1;
+    const float* W3 = h2 > 0 ? b2 + h2 : W2;
+    const float* b3 = W3 + 2 * (size_t)hl;
     T.off_b1[i] = (uint32_t)img.size();
     img.resize(img.size() + b1_bytes, 0);
     for (int j = 0; j < h1; ++j) {
-      auto put = [&](int k, double v) {
-        const uint16_t b = f2bf((float)v);
-        std::memcpy(img.data() + T.off_b1[i] + umma_off(j, k, T.k1), &b, 2);
-      };
-      for (int k = 0; k < dl; ++k) put(k, W1[(size_t)j * din + k]);
+      for (int k = 0; k < dl; ++k) put(T.off_b1[i], j, k, T.k1, W1[(size_t)j * din + k]);
       // A1 carries the scaled aggregate (hi and lo parts), so these columns hold W1 as is;
       // the constant-1 column carries b1 plus the weight of the constant feature N * s_3
       for (int q = 0; q < 3; ++q) {
-        put(T.dle + q, W1[(size_t)j * din + dl + q]);
-        put(T.dle + 4 + q, W1[(size_t)j * din + dl + q]);
+        put(T.off_b1[i], j, T.dle + q, T.k1, W1[(size_t)j * din + dl + q]);
+        put(T.off_b1[i], j, T.dle + 4 + q, T.k1, W1[(size_t)j * din + dl + q]);
       }
-      put(T.dle + 3, (double)b1[j] + (double)W1[(size_t)j * din + dl + 3] * s3 * N);
+      put(T.off_b1[i], j, T.dle + 3, T.k1, (double)b1[j] + (double)W1[(size_t)j * din + dl + 3] * s3 * N);
     }
     T.off_b2[i] = (uint32_t)img.size();
     img.resize(img.size() + b2_bytes, 0);
-    for (int j = 0; j < h2; ++j)
-      for (int k = 0; k < h1; ++k) {
-        const uint16_t b = f2bf(W2[(size_t)j * h1 + k]);
-        std::memcpy(img.data() + T.off_b2[i] + umma_off(j, k, h1), &b, 2);
-      }
+    for (int j = 0; j < h2; ++j) {
+      for (int k = 0; k < h1; ++k) put(T.off_b2[i], j, k, k2, W2[(size_t)j * h1 + k]);
+      put_bias(T.off_b2[i], j, h1, k2, b2[j]);
+    }
     T.off_b3[i] = (uint32_t)img.size();
     img.resize(img.size() + b3_bytes, 0);
     for (int k = 0; k < hl; ++k) {
-      const uint16_t bt = f2bf(W3[k]), bl = f2bf(W3[hl + k]);
-      std::memcpy(img.data() + T.off_b3[i] + umma_off(i, k, hl), &bt, 2);
-      std::memcpy(img.data() + T.off_b3[i] + umma_off(T.n3 / 2 + i, k, hl), &bl, 2);
+      put(T.off_b3[i], i, k, k3, W3[k]);
+      put(T.off_b3[i], T.n3 / 2 + i, k, k3, W3[hl + k]);
     }
+    put_bias(T.off_b3[i], i, hl, k3, b3[0]);
+    put_bias(T.off_b3[i], T.n3 / 2 + i, hl, k3, b3[1]);
   }
   img.resize(round_up((int)img.size(), 16), 0);
   T.img_bytes = (uint32_t)img.size();
 
-  // local-feature words, biases
+  // local-feature words
   const int sumK = c->sumK;
   std::vector<float> x((size_t)sumK * dl);
   e = cudaMemcpy(x.data(), P.x, sizeof(float) * x.size(), cudaMemcpyDeviceToHost);
@@ -640,31 +691,16 @@ mf_status tc_prepare(mf_ctx* c) {
   for (int r = 0; r < sumK; ++r)
     for (int k = 0; k < dl; ++k)
       xw[(size_t)r * T.kw + k / 2] |= (uint32_t)f2bf(x[(size_t)r * dl + k]) << (16 * (k & 1));
-  std::vector<float> b2v((size_t)N * h2), b3v((size_t)N * 2);
-  for (int i = 0; i < N; ++i) {
-    const float* src = w.data() + (size_t)i * P.per_model;
-    const float* b2 = src + (size_t)h1 * din + h1 + (size_t)h2 * h1;
-    for (int j = 0; j < h2; ++j) b2v[(size_t)i * h2 + j] = b2[j];
-    const float* b3 = src + (size_t)h1 * din + h1 + (h2 > 0 ? (size_t)h2 * h1 + h2 : 0) + 2 * (size_t)hl;
-    b3v[2 * i] = b3[0];
-    b3v[2 * i + 1] = b3[1];
-  }
   const size_t o_xw = round_up((int)img.size(), 256);
-  const size_t o_b2 = o_xw + round_up((int)(xw.size() * 4), 256);
-  const size_t o_b3 = o_b2 + round_up((int)(b2v.size() * 4) + 4, 256);
-  const size_t total = o_b3 + round_up((int)(b3v.size() * 4), 256);
+  const size_t total = o_xw + round_up((int)(xw.size() * 4), 256);
   MF_CUDA(cudaMalloc(&c->d_tc, total));
   c->tc_bytes = total;
   unsigned char* base = static_cast<unsigned char*>(c->d_tc);
   MF_CUDA(cudaMemcpy(base, img.data(), img.size(), cudaMemcpyHostToDevice));
   MF_CUDA(cudaMemcpy(base + o_xw, xw.data(), xw.size() * 4, cudaMemcpyHostToDevice));
-  if (!b2v.empty()) MF_CUDA(cudaMemcpy(base + o_b2, b2v.data(), b2v.size() * 4, cudaMemcpyHostToDevice));
-  MF_CUDA(cudaMemcpy(base + o_b3, b3v.data(), b3v.size() * 4, cudaMemcpyHostToDevice));
-  c->stats.h2d_bytes_create += img.size() + xw.size() * 4 + b2v.size() * 4 + b3v.size() * 4;
+  c->stats.h2d_bytes_create += img.size() + xw.size() * 4;
   T.img = base;
   T.xw = reinterpret_cast<const uint32_t*>(base + o_xw);
-  T.b2 = reinterpret_cast<const float*>(base + o_b2);
-  T.b3 = reinterpret_cast<const float*>(base + o_b3);
   MF_CUDA(cudaFuncSetAttribute(k_score_tc<kTcRange>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit));
   MF_CUDA(cudaFuncSetAttribute(k_score_tc<kTcList>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit));
   layout_smem(P, T, 0);
@@ -681,6 +717,13 @@ mf_status tc_search_chunk(mf_ctx* c, const RangeArgs& a, cudaStream_t s) {
   if (T.sm_total > kSmemLimit) {
     set_error("tensor-core path: top-k lists do not fit shared memory; use a smaller k");
     return MF_EUNSUPPORTED;
+  }
+  // digits of the per-tile index stride (grid x pipes x 128), modulo |Lambda|
+  const uint64_t stride = ((uint64_t)c->num_sms * T.pipes * 128) % c->P.total;
+  uint64_t v = stride;
+  for (int i = c->P.n_models - 1; i >= 0; --i) {
+    T.step[i] = (uint32_t)(v % (uint64_t)c->P.K[i]);
+    v /= (uint64_t)c->P.K[i];
   }
   const uint32_t smem = T.sm_total > kSmemFloor ? T.sm_total : kSmemFloor;
   TcList L{};

@@ -40,13 +40,12 @@ struct TcArgs {
   const void* img;                    // bf16 B operands, UMMA K-major no-swizzle layout
   uint32_t img_bytes;
   const uint32_t* xw;                 // [sumK][kw] bf16 pairs of the local features
-  const float* b2;                    // [N][h2]
-  const float* b3;                    // [N][2]
   int32_t k1, kw, h1, h2, hl, n3, dle;
   uint32_t off_b1[MF_MAX_MODELS], off_b2[MF_MAX_MODELS], off_b3[MF_MAX_MODELS];  // bytes in img
-  int32_t pipes, col_d, col_h, col_a, col_d3, pipe_stride;  // TMEM columns
-  uint32_t sm_xw, sm_dem, sm_b2, sm_b3, sm_topk, sm_bar, sm_total;  // shared-memory byte offsets
+  int32_t pipes, col_d, col_h, col_ones, col_a, col_d3, pipe_stride;  // TMEM columns
+  uint32_t sm_xw, sm_dem, sm_rows, sm_desc, sm_topk, sm_bar, sm_total;  // shared-memory byte offsets
   int32_t kcap;                       // per-pipeline list length the layout was sized for
+  uint32_t step[MF_MAX_MODELS];       // mixed-radix digits of the per-tile index stride (range mode)
 };
 
 // Device status bits.
