@@ -50,13 +50,14 @@ __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
 }
 
+// Suspends the thread until the phase completes or about 1 ms passes.
 __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
-      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n"
       " selp.u32 %0, 1, 0, p;\n}"
       : "=r"(ok)
-      : "r"(smem_u32(bar)), "r"(parity)
+      : "r"(smem_u32(bar)), "r"(parity), "r"(1000000u)
       : "memory");
   return ok != 0;
 }
@@ -164,7 +165,7 @@ __device__ __forceinline__ void tmem_st_x16(uint32_t taddr, const uint32_t (&v)[
 // ---------------------------------------------------------------------------
 enum { kTcRange = 0, kTcList = 1 };
 constexpr int kTcMaxPipes = 4;
-constexpr uint32_t kWaitLimit = 1u << 26;
+constexpr uint32_t kWaitLimit = 4096;  // suspended retries (~1 ms each at most)
 
 struct TcList {
   const uint64_t* idx;
@@ -192,7 +193,9 @@ struct PipeWait {
   }
 };
 
-template <int MODE>
+// KW: 32-bit words of an A1 row (8 or 16); AWO: word where the aggregate starts, or
+// -1 to take it from T at run time.
+template <int MODE, int KW, int AWO>
 __global__ void __launch_bounds__(kTcMaxPipes * 128, 1)
 k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   extern __shared__ __align__(1024) unsigned char smem[];
@@ -381,27 +384,27 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
       aw[2] = l0 | (l1 << 16);
       aw[3] = l2;
     }
-    const int awo = T.dle >> 1;
+    // A1 row = option-table words with the aggregate words at word awo (the table holds
+    // zeros there)
+    const int awo = AWO >= 0 ? AWO : (T.dle >> 1);
+    auto word = [&](int j, uint32_t x) -> uint32_t {
+      if (AWO >= 0) return (j >= AWO && j < AWO + 4) ? aw[(j - AWO) & 3] : x;
+      const int a = j - awo;
+      return a == 0 ? aw[0] : a == 1 ? aw[1] : a == 2 ? aw[2] : a == 3 ? aw[3] : x;
+    };
     auto write_a1 = [&](int i) {
-      const uint4* src = xw_s + (size_t)rows[i * 128 + row] * (T.kw >> 2);
-      // word j: local-feature pair, or aggregate word j - awo for awo <= j < awo + 4
-      auto pick = [&](int j, uint32_t x) -> uint32_t {
-        const int a = j - awo;
-        return a == 0 ? aw[0] : a == 1 ? aw[1] : a == 2 ? aw[2] : a == 3 ? aw[3] : x;
-      };
-      if (T.kw == 8) {
-        const uint4 q0 = src[0], q1 = src[1];
-        uint32_t v[8] = {pick(0, q0.x), pick(1, q0.y), pick(2, q0.z), pick(3, q0.w),
-                         pick(4, q1.x), pick(5, q1.y), pick(6, q1.z), pick(7, q1.w)};
-        tmem_st_x8(tA + lane_off, v);
-      } else {
-        const uint4 q0 = src[0], q1 = src[1], q2 = src[2], q3 = src[3];
-        uint32_t v[16] = {pick(0, q0.x),  pick(1, q0.y),  pick(2, q0.z),  pick(3, q0.w),
-                          pick(4, q1.x),  pick(5, q1.y),  pick(6, q1.z),  pick(7, q1.w),
-                          pick(8, q2.x),  pick(9, q2.y),  pick(10, q2.z), pick(11, q2.w),
-                          pick(12, q3.x), pick(13, q3.y), pick(14, q3.z), pick(15, q3.w)};
-        tmem_st_x16(tA + lane_off, v);
+      const uint4* src = xw_s + (size_t)rows[i * 128 + row] * (KW >> 2);
+      uint32_t v[KW];
+#pragma unroll
+      for (int q = 0; q < KW / 4; ++q) {
+        const uint4 w4 = src[q];
+        v[4 * q + 0] = word(4 * q + 0, w4.x);
+        v[4 * q + 1] = word(4 * q + 1, w4.y);
+        v[4 * q + 2] = word(4 * q + 2, w4.z);
+        v[4 * q + 3] = word(4 * q + 3, w4.w);
       }
+      if constexpr (KW == 8) tmem_st_x8(tA + lane_off, v);
+      else tmem_st_x16(tA + lane_off, v);
     };
 
     write_a1(0);
@@ -581,6 +584,18 @@ void layout_smem(const Params& P, TcArgs& T, int kcap) {
 }
 
 constexpr uint32_t kSmemLimit = 227 * 1024 - 1024;  // static shared variables take the rest
+
+using TcFn = void (*)(const Params, const TcArgs, const RangeArgs, const TcList);
+
+// Instantiation for the A1 row shape: d_L = 8 and d_L = 16 have fixed word layouts.
+TcFn tc_kernel(int mode, const TcArgs& T) {
+  if (mode == kTcRange) {
+    if (T.kw == 8) return T.dle == 8 ? k_score_tc<kTcRange, 8, 4> : k_score_tc<kTcRange, 8, -1>;
+    return T.dle == 16 ? k_score_tc<kTcRange, 16, 8> : k_score_tc<kTcRange, 16, -1>;
+  }
+  if (T.kw == 8) return T.dle == 8 ? k_score_tc<kTcList, 8, 4> : k_score_tc<kTcList, 8, -1>;
+  return T.dle == 16 ? k_score_tc<kTcList, 16, 8> : k_score_tc<kTcList, 16, -1>;
+}
 constexpr uint32_t kSmemFloor = 120 * 1024;          // keeps one CTA (one TMEM owner) per SM
 
 }  // namespace
@@ -701,8 +716,8 @@ mf_status tc_prepare(mf_ctx* c) {
   c->stats.h2d_bytes_create += img.size() + xw.size() * 4;
   T.img = base;
   T.xw = reinterpret_cast<const uint32_t*>(base + o_xw);
-  MF_CUDA(cudaFuncSetAttribute(k_score_tc<kTcRange>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit));
-  MF_CUDA(cudaFuncSetAttribute(k_score_tc<kTcList>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit));
+  MF_CUDA(cudaFuncSetAttribute(tc_kernel(kTcRange, T), cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit));
+  MF_CUDA(cudaFuncSetAttribute(tc_kernel(kTcList, T), cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit));
   layout_smem(P, T, 0);
   if (T.sm_total > kSmemLimit) {
     set_error("tensor-core path: tables and weights exceed shared memory");
@@ -727,7 +742,7 @@ mf_status tc_search_chunk(mf_ctx* c, const RangeArgs& a, cudaStream_t s) {
   }
   const uint32_t smem = T.sm_total > kSmemFloor ? T.sm_total : kSmemFloor;
   TcList L{};
-  k_score_tc<kTcRange><<<c->num_sms, T.pipes * 128, smem, s>>>(c->P, T, a, L);
+  tc_kernel(kTcRange, T)<<<c->num_sms, T.pipes * 128, smem, s>>>(c->P, T, a, L);
   MF_CUDA(cudaGetLastError());
   return MF_OK;
 }
@@ -744,7 +759,7 @@ mf_status tc_score_list(mf_ctx* c, const uint64_t* idx, uint64_t n, float* score
   if (grid > (uint64_t)c->num_sms) grid = c->num_sms;
   RangeArgs R{};
   TcList L{idx, n, score, feas, pred};
-  k_score_tc<kTcList><<<(unsigned)grid, T.pipes * 128, smem, s>>>(c->P, T, R, L);
+  tc_kernel(kTcList, T)<<<(unsigned)grid, T.pipes * 128, smem, s>>>(c->P, T, R, L);
   MF_CUDA(cudaGetLastError());
   return MF_OK;
 }
