@@ -407,10 +407,23 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
       else tmem_st_x16(tA + lane_off, v);
     };
 
+    // The issuing thread alone polls the pipeline's mbarrier; the other threads
+    // wait at the named barrier (no issue slots), which the issuer joins once the
+    // MMAs have completed.
+    auto await_mma = [&]() {
+      if (leader) wait_bar(mbar, phase);
+      phase ^= 1u;
+      named_bar(barid, 128);
+      tc_fence_after();
+    };
+    auto publish = [&]() {  // make this thread's tensor-memory stores visible to the issuer
+      tmem_wait_st();
+      tc_fence_before();
+      named_bar(barid, 128);
+    };
+
     write_a1(0);
-    tmem_wait_st();
-    tc_fence_before();
-    named_bar(barid, 128);
+    publish();
     for (int i = 0; i < N; ++i) {
       if (leader) {
         tc_fence_after();
@@ -418,37 +431,27 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
         issue_mma1(i);
         mma_commit(mbar);
       }
-      wait_bar(mbar, phase);
-      phase ^= 1u;
-      tc_fence_after();
+      await_mma();
       epilogue(T.h1, tH1);  // layer 1 (bias in the constant column)
       if (T.h2 > 0) {
-        tmem_wait_st();
-        tc_fence_before();
-        named_bar(barid, 128);
+        publish();
         if (leader) {
           tc_fence_after();
           issue_mma2(i);
           mma_commit(mbar);
         }
-        wait_bar(mbar, phase);
-        phase ^= 1u;
-        tc_fence_after();
+        await_mma();
         epilogue(T.h2, tH2);  // layer 2 (bias through the ones block)
       }
       if (i + 1 < N) write_a1(i + 1);
-      tmem_wait_st();
-      tc_fence_before();
-      named_bar(barid, 128);
+      publish();
     }
     if (leader) {
       tc_fence_after();
       issue_mma3(N - 1);
       mma_commit(mbar);
     }
-    wait_bar(mbar, phase);
-    phase ^= 1u;
-    tc_fence_after();
+    await_mma();
 
     // ---- final epilogue: per-model outputs, constraints, objective ----
     uint32_t d3[32];
