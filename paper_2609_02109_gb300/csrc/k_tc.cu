@@ -193,9 +193,22 @@ struct PipeWait {
   }
 };
 
+// `steps` MMAs of K = 16 along one K extent; S > 0 unrolls a compile-time count (the
+// issuing thread's instruction stream is on the critical path of every round trip).
+template <int S>
+__device__ __forceinline__ void mma_steps(int steps, uint32_t d_tmem, uint32_t a_tmem, uint64_t desc,
+                                          uint32_t idesc, uint32_t acc0) {
+  if constexpr (S > 0) {
+#pragma unroll
+    for (int s = 0; s < S; ++s) mma_ts(d_tmem, a_tmem + 8u * s, desc + 16u * s, idesc, s > 0 ? 1u : acc0);
+  } else {
+    for (int s = 0; s < steps; ++s) mma_ts(d_tmem, a_tmem + 8u * s, desc + 16u * s, idesc, s > 0 ? 1u : acc0);
+  }
+}
+
 // KW: 32-bit words of an A1 row (8 or 16); AWO: word where the aggregate starts, or
-// -1 to take it from T at run time.
-template <int MODE, int KW, int AWO>
+// -1 to take it from T at run time.  S1, S2, S3: K-steps of the three layers (0 = run time).
+template <int MODE, int KW, int AWO, int S1, int S2, int S3>
 __global__ void __launch_bounds__(kTcMaxPipes * 128, 1)
 k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   extern __shared__ __align__(1024) unsigned char smem[];
@@ -315,18 +328,9 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     for (int i = 0; i < N; ++i) rows[i * 128 + row] = (uint16_t)(P.off[i] + (int)((idx0 / P.stride[i]) % P.K[i]));
   }
 
-  auto issue_mma1 = [&](int i) {
-    const uint64_t d = desc_s[3 * i + 0];
-    for (int s = 0; s < s1; ++s) mma_ts(tD, tA + 8 * s, d + 16u * s, id1, s > 0);
-  };
-  auto issue_mma2 = [&](int i) {
-    const uint64_t d = desc_s[3 * i + 1];
-    for (int s = 0; s < s2; ++s) mma_ts(tD, tH1 + 8 * s, d + 16u * s, id2, s > 0);
-  };
-  auto issue_mma3 = [&](int i) {
-    const uint64_t d = desc_s[3 * i + 2];
-    for (int s = 0; s < s3; ++s) mma_ts(tD3, tH2 + 8 * s, d + 16u * s, id3, (i > 0 || s > 0));
-  };
+  auto issue_mma1 = [&](int i) { mma_steps<S1>(s1, tD, tA, desc_s[3 * i + 0], id1, 0u); };
+  auto issue_mma2 = [&](int i) { mma_steps<S2>(s2, tD, tH1, desc_s[3 * i + 1], id2, 0u); };
+  auto issue_mma3 = [&](int i) { mma_steps<S3>(s3, tD3, tH2, desc_s[3 * i + 2], id3, i > 0 ? 1u : 0u); };
   // fp32 accumulators [0, width) -> ReLU -> bf16 pairs at dst
   auto epilogue = [&](int width, uint32_t dst) {
     for (int c0 = 0; c0 < width; c0 += 32) {
@@ -590,14 +594,18 @@ constexpr uint32_t kSmemLimit = 227 * 1024 - 1024;  // static shared variables t
 
 using TcFn = void (*)(const Params, const TcArgs, const RangeArgs, const TcList);
 
-// Instantiation for the A1 row shape: d_L = 8 and d_L = 16 have fixed word layouts.
+// Instantiations: the two benchmark shapes (d_L 8, 64-64 and d_L 16, 128-128) with all
+// counts fixed at compile time, and a run-time fallback per A1 row width.
+template <int MODE>
+TcFn tc_kernel_mode(const TcArgs& T) {
+  if (T.kw == 8 && T.dle == 8 && T.h1 == 64 && T.h2 == 64) return k_score_tc<MODE, 8, 4, 1, 5, 5>;
+  if (T.kw == 16 && T.dle == 16 && T.h1 == 128 && T.h2 == 128) return k_score_tc<MODE, 16, 8, 2, 9, 9>;
+  if (T.kw == 8) return k_score_tc<MODE, 8, -1, 0, 0, 0>;
+  return k_score_tc<MODE, 16, -1, 0, 0, 0>;
+}
+
 TcFn tc_kernel(int mode, const TcArgs& T) {
-  if (mode == kTcRange) {
-    if (T.kw == 8) return T.dle == 8 ? k_score_tc<kTcRange, 8, 4> : k_score_tc<kTcRange, 8, -1>;
-    return T.dle == 16 ? k_score_tc<kTcRange, 16, 8> : k_score_tc<kTcRange, 16, -1>;
-  }
-  if (T.kw == 8) return T.dle == 8 ? k_score_tc<kTcList, 8, 4> : k_score_tc<kTcList, 8, -1>;
-  return T.dle == 16 ? k_score_tc<kTcList, 16, 8> : k_score_tc<kTcList, 16, -1>;
+  return mode == kTcRange ? tc_kernel_mode<kTcRange>(T) : tc_kernel_mode<kTcList>(T);
 }
 constexpr uint32_t kSmemFloor = 120 * 1024;          // keeps one CTA (one TMEM owner) per SM
 
