@@ -199,7 +199,12 @@ mf_status mf_ga_step(mf_ctx *ctx, const mf_ga_params *g, uint64_t seed, int32_t 
 /* A complete GA decision: init, then g->gens fitness batches with a generation
  * step between consecutive ones; returns the fittest individual of the last
  * population (lowest slot among equals) in best_genome[N] (host) and its
- * fitness.  Synchronous. */
+ * fitness.  Synchronous.  The operators and random draws are those of
+ * mf_ga_init / mf_ga_step.  For fp32 predictors with d_L = 8, h1 = h2 = 64,
+ * N <= 8 and pop <= 8 x the SM count, the whole decision runs as one
+ * cooperative kernel (mf_stats.kernel_launches_last = 1); otherwise as one CUDA
+ * graph of init, fitness and step kernels.  MF_ETIMEOUT if the cooperative
+ * kernel's grid barrier gave up waiting (the result is then not valid). */
 mf_status mf_ga_run(mf_ctx *ctx, const mf_ga_params *g, uint64_t seed, int32_t *best_genome,
                     float *best_fitness, void *stream);
 

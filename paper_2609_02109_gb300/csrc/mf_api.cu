@@ -489,7 +489,12 @@ mf_status mf_ga_run(mf_ctx* ctx, const mf_ga_params* g, uint64_t seed, int32_t* 
   if (!best_genome || !best_fitness) return einval("NULL output");
   DeviceGuard guard(ctx->device);
   cudaStream_t s = (cudaStream_t)stream;
-  st = ga_run_graph(ctx, g, seed, s);
+  int launches = 1;  // one cooperative kernel
+  st = ga_run_persistent(ctx, g, seed, s);
+  if (st == MF_EUNSUPPORTED) {
+    st = ga_run_graph(ctx, g, seed, s);
+    launches = 2 + g->gens * 2 + (g->gens - 1);  // init, (wide + combine) x gens, steps, best
+  }
   if (st != MF_OK) return st;
   const int N = ctx->P.n_models;
   int32_t* h_g = (int32_t*)ctx->h_stage;
@@ -498,10 +503,14 @@ mf_status mf_ga_run(mf_ctx* ctx, const mf_ga_params* g, uint64_t seed, int32_t* 
   MF_CUDA(cudaMemcpyAsync(h_g, ctx->d_ga_out, sizeof(int32_t) * N + sizeof(float), cudaMemcpyDeviceToHost, s));
   st = read_status(ctx, s, h_status, true);
   if (st != MF_OK) return st;
+  if (*h_status & kStatusTimeout) {
+    g_last_error = "the GA kernel's grid barrier gave up waiting";
+    return MF_ETIMEOUT;
+  }
   std::memcpy(best_genome, h_g, sizeof(int32_t) * N);
   *best_fitness = *h_f;
   ctx->stats.d2h_bytes_last = sizeof(int32_t) * N + sizeof(float) + sizeof(uint32_t);
-  ctx->stats.kernel_launches_last = 2 + g->gens * 2 + (g->gens - 1);  // init, (wide + combine) x gens, steps, best
+  ctx->stats.kernel_launches_last = launches;
   return MF_OK;
 }
 

@@ -274,5 +274,8 @@ mf_status ga_best(mf_ctx* c, const int32_t* pop, const float* fit, int P, int32_
 // Whole GA decision as one CUDA graph launch on `s`; the result lands in c->d_ga_out
 // and the pinned staging buffer is sized for it.
 mf_status ga_run_graph(mf_ctx* c, const mf_ga_params* g, uint64_t seed, cudaStream_t s);
+// Whole GA decision in one cooperative kernel; MF_EUNSUPPORTED (nothing launched) when
+// the shape or the device does not allow it.
+mf_status ga_run_persistent(mf_ctx* c, const mf_ga_params* g, uint64_t seed, cudaStream_t s);
 
 }  // namespace mf

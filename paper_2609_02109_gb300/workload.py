@@ -179,6 +179,51 @@ def stress(seed: int = 4, precision="bf16", **kw) -> dict:
                         soft_penalty=0.1, precision=precision, **kw)
 
 
+def _ints(seed: int, purpose: int, model: int, n: int, lo: int, hi: int) -> np.ndarray:
+    """n integers uniform on [lo, hi] (multiply-shift on the top 32 bits), as float32."""
+    z = stream_u64(stream_key(seed, purpose, model), n) >> np.uint64(32)
+    span = np.uint64(hi - lo + 1)
+    return ((z * span) >> np.uint64(32)).astype(np.int64).astype(np.float32) + np.float32(lo)
+
+
+def integer_landscape(n_options, seed: int, vram_cap: float, objective="weighted_thr",
+                      soft_penalty=0.0) -> dict:
+    """A d_L = 8, 12->64->64->2 problem whose every input is a small integer.
+
+    Local features in [-2, 2], demands in [1, 9] (three columns), W1 in [-1, 1]
+    with zero columns for the four aggregate inputs, W2 and W3 in [-1, 1], biases
+    in [-2, 2], SLA ceilings and objective weights small integers.  Every
+    intermediate value of the predictor and the objective is then an integer
+    below 2**24 in magnitude, so fp32 and fp64 evaluation in any summation order
+    give the same number and a GA run is reproducible bit for bit across
+    implementations.
+    """
+    n_options = np.asarray(n_options, dtype=np.int32)
+    n = int(n_options.size)
+    d, h, d_in = 8, 64, 12
+    locs, dems, ws = [], [], []
+    for i in range(n):
+        k = int(n_options[i])
+        locs.append(_ints(seed, P_LOCAL, i, k * d, -2, 2).reshape(k, d))
+        dems.append(np.stack([_ints(seed, P_SM, i, k, 1, 9), _ints(seed, P_VRAM, i, k, 1, 9),
+                              _ints(seed, P_BW, i, k, 1, 9)], axis=1))
+        w1 = _ints(seed, P_W1, i, h * d_in, -1, 1).reshape(h, d_in)
+        w1[:, d:] = 0.0
+        ws.append(np.concatenate([w1.ravel(), _ints(seed, P_B1, i, h, -2, 2),
+                                  _ints(seed, P_W2, i, h * h, -1, 1), _ints(seed, P_B2, i, h, -2, 2),
+                                  _ints(seed, P_W3, i, 2 * h, -1, 1), _ints(seed, P_B3, i, 2, -2, 2)]))
+    return dict(
+        n_options=n_options, d_local=d, hidden1=h, hidden2=h,
+        local_feats=np.ascontiguousarray(np.concatenate(locs, axis=0), dtype=np.float32),
+        demand=np.ascontiguousarray(np.concatenate(dems, axis=0), dtype=np.float32),
+        weights=np.ascontiguousarray(np.concatenate(ws), dtype=np.float32),
+        agg_scale=default_agg_scale(n), vram_cap=float(vram_cap),
+        soft_penalty=float(soft_penalty), objective=objective, out_act="identity", precision="fp32",
+        sla=_ints(seed, P_SLA, 0, n, 40, 120), obj_w=_ints(seed, P_OBJW, 0, n, 1, 3),
+        scenario_seed=int(seed),
+    )
+
+
 GA_SCENARIO_SEEDS = tuple(range(100, 108))
 GA_RUN_SEEDS = tuple(range(1000, 1050))
 

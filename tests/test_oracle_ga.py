@@ -138,3 +138,33 @@ def test_ga_finds_optimum_of_tiny_space(oracle_mod):
     J, genome = o.ga_run(_ga(pop=64, gens=30), seed=1000)
     assert J == ts[0]
     assert list(genome) == list(o.decode(int(ti[0])))
+
+
+@pytest.mark.parametrize("opts,seed,cap", [([12, 9, 9, 9, 9], 5, 30.0), ([5] * 8, 7, 45.0)])
+def test_integer_landscape_is_exact_in_any_order(oracle_mod, opts, seed, cap):
+    """The premise of the bit-exact GA tests on the GPU: in the integer landscapes
+    every input is an integer and the largest value any partial sum can reach is
+    below 2**24, so fp32 arithmetic is exact whatever the summation order."""
+    prob = W.integer_landscape(opts, seed, cap, objective="soft_lat", soft_penalty=0.5)
+    n, d, h = len(opts), 8, 64
+    per = W.param_count(d, h, h)
+    for a in (prob["local_feats"], prob["demand"], prob["weights"], prob["sla"], prob["obj_w"]):
+        assert np.all(a == np.round(a))
+    w = prob["weights"].reshape(n, per).astype(np.float64)
+    x = float(np.abs(prob["local_feats"]).max())
+    b1 = h * (d + 4)
+    for i in range(n):
+        W1 = w[i, :b1].reshape(h, d + 4)
+        assert np.all(W1[:, d:] == 0)  # the aggregate inputs do not enter
+        h1 = d * x * np.abs(W1).max() + np.abs(w[i, b1:b1 + h]).max()
+        o2 = b1 + h
+        h2 = h * h1 * np.abs(w[i, o2:o2 + h * h]).max() + np.abs(w[i, o2 + h * h:o2 + h * h + h]).max()
+        o3 = o2 + h * h + h
+        out = h * h2 * np.abs(w[i, o3:o3 + 2 * h]).max() + np.abs(w[i, o3 + 2 * h:]).max()
+        bound_J = n * (float(prob["obj_w"].max()) * out + 0.5 * (out + float(np.abs(prob["sla"]).max())))
+        assert bound_J < 2 ** 24
+    o = oracle_mod.Oracle(prob)
+    idx = np.random.default_rng(1).integers(0, o.space_size(), 3000).astype(np.uint64)
+    s, f, pred, _ = o.score_list(idx, with_pred=True)
+    assert np.all(pred == np.round(pred))
+    assert f.any() and np.all(2 * s[f] == np.round(2 * s[f]))  # soft penalty 0.5: halves
