@@ -211,97 +211,258 @@ mf_status ga_run_graph(mf_ctx* c, const mf_ga_params* g, uint64_t seed, cudaStre
 // ---------------------------------------------------------------------------
 // Whole GA decision in one cooperative kernel (fp32 predictors d_L 8, 64-64).
 //
-// Each CTA owns a slice of at most kGaMaxSlice individuals.  One thread per
-// (model m, hidden unit j) keeps row j of W1 and W2 of model m in registers for
-// the whole run and evaluates that unit for every individual of the slice, so a
-// weight is read once per run, not once per individual.  Per generation:
-//   aggregate -> layer 1 -> layers 2 and 3 -> objective and constraints of the
-//   slice -> grid barrier -> the generation's population and fitness copied
-//   from L2 into shared memory in one pass -> the slice's children (elite,
-//   tournaments, crossover, mutation: the operators and draws of k_ga_step)
-// Population and fitness are double-buffered in global memory.  A buffer written
-// in generation g + 2 was last read (copied to shared memory) in generation g,
-// before its reader arrived at the barrier that ends generation g + 1, which the
-// writer has passed.
+// CTA b owns the slice [8b, 8b + 8) of the population.  Thread (model m, hidden
+// unit j) keeps rows j of W1 and W2 in registers for the whole run, so a weight is
+// read from memory once per run.  One generation:
+//   layer 1    thread (m, j) for the slice's candidates
+//   layer 2-3  thread (m, j) for all 8 candidates (each shared-memory load of four
+//              layer-1 activations is one broadcast to the warp); layer 3 sums over
+//              the warp in butterfly shuffles where each step halves the values a
+//              lane carries
+//   objective  warp c for candidate c, lane i for model i (Eq. 7-9)
+//   step       warp c breeds child 8b + c: lane t holds tournament entry t and
+//              fetches its fitness and genome; the winners' genomes come by
+//              shuffle; lane i mutates gene i and adds its demand to the child's
+//              aggregate state.  The elite (slot 0) is the best of the CTAs' bests.
+// There is no grid-wide barrier.  Every value another CTA reads -- an individual's
+// fitness, the two halves of its genome (gene i in byte i mod 4), a CTA's best --
+// is a 64-bit word whose high half is the tag g + 1 of its generation g, written
+// and read as single 64-bit accesses.  A reader spins on exactly the words it
+// needs until their tags match, so each generation waits only for the CTAs whose
+// individuals its tournaments drew (and CTA 0, for the elite, for every CTA's
+// best).  The words live in a ring of R = min(gens + 1, kGaRingMax) generations;
+// before a CTA writes generation g + 1 over g + 1 - R it checks that every CTA has
+// finished reading that generation (per-CTA progress counters, read ahead of use).
+// Every operator and draw is that of k_ga_step, so the run equals init + (fitness,
+// step) x gens up to the fp32 rounding of the fitness.  Every spin gives up after
+// kGaSpinLimit polls, sets the timeout bit of the status word and ends the CTA.
 // ---------------------------------------------------------------------------
 namespace mf {
 
 constexpr int kGaMaxSlice = 8;
-constexpr uint32_t kGridPollLimit = 1u << 22;  // polls of about a microsecond: a few seconds
+constexpr int kGaRingMax = 128;                // generations held in the ring (at most)
+constexpr uint32_t kGaSpinLimit = 1u << 22;    // polls of about a microsecond: a few seconds
+
+struct __align__(32) GaRec {   // one individual of one generation
+  unsigned long long fw;       // tag | fitness bits
+  unsigned long long glo;      // tag | genes 0-3
+  unsigned long long ghi;      // tag | genes 4-7
+  unsigned long long pad;
+};
+
+struct __align__(32) GaBest {  // fittest individual of one CTA's slice
+  unsigned long long fw;       // tag | fitness bits
+  unsigned long long sw;       // tag | slot
+  unsigned long long glo, ghi;
+};
 
 struct GaPersist {
-  int32_t* pop0;
-  int32_t* pop1;
-  float* fit0;           // fitness of even generations
-  float* fit1;           // fitness of odd generations
-  unsigned int* flags;   // [ctas] last epoch each CTA reached
+  GaRec* rec;            // [ring][pop]
+  GaBest* best;          // [ring][ctas]
+  unsigned int* prog;    // [ctas] generations whose records the CTA has finished reading
   int32_t* out_genome;
   float* out_fit;
   const uint64_t* seed;
   int gens;
-  int slice;
+  int ring;
 };
 
-__device__ __forceinline__ unsigned int ld_acquire_gpu(const unsigned int* p) {
-  unsigned int v;
-  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+// fma.rn.f32x2: two fp32 fused multiply-adds (each rounded as fmaf) in one instruction.
+__device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
+  unsigned long long r;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;"
+      : "=l"(r)
+      : "l"(*reinterpret_cast<unsigned long long*>(&a)), "l"(*reinterpret_cast<unsigned long long*>(&b)),
+        "l"(*reinterpret_cast<unsigned long long*>(&c)));
+  return *reinterpret_cast<float2*>(&r);
+}
+
+__device__ __forceinline__ unsigned long long ld_word(const unsigned long long* p) {
+  unsigned long long v;
+  asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
   return v;
 }
 
-__device__ __forceinline__ void st_release_gpu(unsigned int* p, unsigned int v) {
-  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+__device__ __forceinline__ void st_word(unsigned long long* p, unsigned long long v) {
+  asm volatile("st.relaxed.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
 }
 
-// Grid barrier: every CTA publishes `epoch` in its own flag, then polls all flags
-// (one per thread).  Gives up after kGridPollLimit polls, flags the status word and
-// lets the kernel run to its end.
-__device__ void grid_barrier(unsigned int* flags, unsigned int nblocks, unsigned int epoch, uint32_t* status) {
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    __threadfence();
-    st_release_gpu(flags + blockIdx.x, epoch);
+__device__ __forceinline__ unsigned int ld_u32(const unsigned int* p) {
+  unsigned int v;
+  asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ void st_u32(unsigned int* p, unsigned int v) {
+  asm volatile("st.relaxed.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ unsigned long long tagged(uint32_t tag, uint32_t payload) {
+  return ((unsigned long long)tag << 32) | payload;
+}
+
+__device__ __forceinline__ bool has_tag(unsigned long long w, uint32_t tag) {
+  return (uint32_t)(w >> 32) == tag;
+}
+
+// (fitness, slot) maximum over the warp: higher fitness, then lower slot; slot < 0 is empty.
+__device__ __forceinline__ void warp_best(float& f, int& s) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float of = __shfl_xor_sync(0xffffffffu, f, o);
+    const int os = __shfl_xor_sync(0xffffffffu, s, o);
+    if (os >= 0 && (s < 0 || of > f || (of == f && os < s))) { f = of; s = os; }
   }
-  uint32_t n = 0;
-  while (true) {
-    bool mine = true;
-    for (unsigned int q = threadIdx.x; q < nblocks; q += blockDim.x)
-      mine = mine && (ld_acquire_gpu(flags + q) >= epoch);
-    if (__syncthreads_and(mine)) break;
-    if (++n > kGridPollLimit) {
-      if (threadIdx.x == 0) atomicOr(status, kStatusTimeout);
-      break;
+}
+
+// One butterfly step that halves the values a lane carries: the two lanes that
+// differ in `bit` each keep one half, so afterwards v[i] (i < n) is the pair's sum
+// of value i + n * (that lane bit).
+template <int n>
+__device__ __forceinline__ void fold(float* v, int bit) {
+  const bool b = (threadIdx.x >> bit) & 1;
+#pragma unroll
+  for (int i = 0; i < n; ++i) {
+    const float send = b ? v[i] : v[i + n];
+    const float keep = b ? v[i + n] : v[i];
+    v[i] = keep + __shfl_xor_sync(0xffffffffu, send, 1 << bit);
+  }
+}
+
+// Spin until the three words of record r carry `tag` (or the poll limit); false on timeout.
+__device__ __forceinline__ bool fetch_rec(const GaRec* r, uint32_t tag, float& f, uint32_t& lo, uint32_t& hi) {
+  for (uint32_t n = 0; n < kGaSpinLimit; ++n) {
+    const unsigned long long a = ld_word(&r->fw), b = ld_word(&r->glo), c = ld_word(&r->ghi);
+    if (has_tag(a, tag) && has_tag(b, tag) && has_tag(c, tag)) {
+      f = __uint_as_float((uint32_t)a);
+      lo = (uint32_t)b;
+      hi = (uint32_t)c;
+      return true;
     }
   }
+  return false;
 }
 
-template <int DL, int MAXT>
+// Fittest of the CTAs' bests of one generation, on every lane of the warp; false on timeout.
+__device__ bool best_of_ctas(const GaBest* bst, int n, uint32_t tag, float& f, int& s, uint32_t& lo,
+                             uint32_t& hi) {
+  const int lane = threadIdx.x & 31;
+  f = -INFINITY;
+  s = -1;
+  lo = hi = 0;
+  bool ok = true;
+  for (int b = lane; b < n && ok; b += 32) {
+    ok = false;
+    for (uint32_t it = 0; it < kGaSpinLimit; ++it) {
+      const GaBest* r = bst + b;
+      const unsigned long long a = ld_word(&r->fw), w = ld_word(&r->sw), x = ld_word(&r->glo),
+                               y = ld_word(&r->ghi);
+      if (has_tag(a, tag) && has_tag(w, tag) && has_tag(x, tag) && has_tag(y, tag)) {
+        const float rf = __uint_as_float((uint32_t)a);
+        const int rs = (int)(uint32_t)w;
+        if (s < 0 || rf > f || (rf == f && rs < s)) { f = rf; s = rs; lo = (uint32_t)x; hi = (uint32_t)y; }
+        ok = true;
+        break;
+      }
+    }
+  }
+  ok = __all_sync(0xffffffffu, ok);
+  const int mine = s;
+  warp_best(f, s);
+  const unsigned int src = __ffs(__ballot_sync(0xffffffffu, mine == s)) - 1;
+  lo = __shfl_sync(0xffffffffu, lo, src);
+  hi = __shfl_sync(0xffffffffu, hi, src);
+  return ok;
+}
+
+// Random numbers of one child that do not depend on fitness (lane = tournament
+// entry t for t < 32, lane = gene i for i < N).
+struct ChildDraws {
+  int ta, tb;      // tournament A / B entry `lane` (-1: none)
+  int take_b;      // gene `lane` comes from parent B
+  int mutate;      // gene `lane` mutates
+  int mval;        // ... to this option
+};
+
+__device__ __forceinline__ ChildDraws child_draws(const GaArgs& g, uint64_t sd, uint32_t G, uint32_t c,
+                                                  int lane, int N, int myK) {
+  ChildDraws d;
+  d.ta = d.tb = -1;
+  d.take_b = d.mutate = d.mval = 0;
+  if (lane < g.tournament) {
+    d.ta = ga_unif(ga_rng(sd, G, c, kGaTourA, (uint32_t)lane), (uint32_t)g.pop);
+    d.tb = ga_unif(ga_rng(sd, G, c, kGaTourB, (uint32_t)lane), (uint32_t)g.pop);
+  }
+  if (lane < N) {
+    d.take_b = (int)(ga_rng(sd, G, c, kGaCross, (uint32_t)lane) >> 63);
+    d.mutate = (uint32_t)(ga_rng(sd, G, c, kGaMut, (uint32_t)lane) >> 40) < g.mut_thr;
+    if (d.mutate) d.mval = ga_unif(ga_rng(sd, G, c, kGaMutVal, (uint32_t)lane), (uint32_t)myK);
+  }
+  return d;
+}
+
+// Winner of one tournament and its genome halves.  Lane t < 32 holds entry t (slot s,
+// -1 for none) with its fitness and genome; entries 32.. are fetched here.
+__device__ __forceinline__ bool tournament_winner(const GaArgs& g, uint64_t sd, uint32_t G, uint32_t c,
+                                                  uint32_t purpose, const GaRec* rec, uint32_t tag, int s,
+                                                  float f, uint32_t& lo, uint32_t& hi) {
+  const int lane = threadIdx.x & 31;
+  bool ok = true;
+  for (int t = lane + 32; t < g.tournament && ok; t += 32) {  // tournaments larger than a warp
+    const int x = ga_unif(ga_rng(sd, G, c, purpose, (uint32_t)t), (uint32_t)g.pop);
+    float v;
+    uint32_t xl, xh;
+    ok = fetch_rec(rec + x, tag, v, xl, xh);
+    if (ok && (s < 0 || v > f || (v == f && x < s))) { f = v; s = x; lo = xl; hi = xh; }
+  }
+  ok = __all_sync(0xffffffffu, ok);
+  const int mine = s;
+  warp_best(f, s);
+  const unsigned int src = __ffs(__ballot_sync(0xffffffffu, mine == s)) - 1;
+  lo = __shfl_sync(0xffffffffu, lo, src);
+  hi = __shfl_sync(0xffffffffu, hi, src);
+  return ok;
+}
+
+// a[i] for a per-model array of the kernel parameters, read with constant indices
+// (a runtime index into a parameter array would copy it to local memory)
+template <typename T>
+__device__ __forceinline__ T pick(const T (&a)[MF_MAX_MODELS], int i) {
+  T v = a[0];
+#pragma unroll
+  for (int k = 1; k < MF_MAX_MODELS; ++k) v = k == i ? a[k] : v;
+  return v;
+}
+
+template <int MAXT>
 __global__ void __launch_bounds__(MAXT, 1)
 k_ga_persist(const Params P, const GaArgs g, const GaPersist G) {
-  constexpr int H = 64, DIN = DL + 4, SM = kGaMaxSlice;
+  constexpr int H = 64, DL = 8, DIN = DL + 4, SM = kGaMaxSlice;
+  constexpr int WPM = H / 32;         // warps per model
   extern __shared__ __align__(16) float sm[];
+  __shared__ int s_abort;
+  __shared__ float s_fit[SM];
+  __shared__ uint32_t s_glo[SM], s_ghi[SM];
   const int N = P.n_models;
-  const int sumK = P.off[N - 1] + P.K[N - 1];
+  const int sumK = pick(P.off, N - 1) + pick(P.K, N - 1);
   const int pop = g.pop;
-  const int pop4 = (pop + 3) & ~3;
   // shared memory; every float region is a multiple of 4 floats so the float4 rows align
   float* sh1 = sm;                                           // [N][SM][H] layer-1 activations
-  float* spart = sh1 + (size_t)N * SM * H;                   // [2][SM][N][2] layer-3 halves
-  float* sagg = spart + 4 * SM * N;                          // [SM][4] scaled aggregate, raw VRAM
-  float* sb3 = sagg + 4 * SM;                                // [MF_MAX_MODELS][2]
-  float* sfit = sb3 + 2 * MF_MAX_MODELS;                     // [pop] fitness of the generation
-  float* sx = sfit + pop4;                                   // [sumK][DL] local features
+  float* spart = sh1 + (size_t)N * SM * H;                   // [WPM][SM][N][2] layer-3 warp sums
+  float* sagg = spart + (size_t)WPM * SM * N * 2;            // [SM][4] scaled aggregate, raw VRAM
+  float* sx = sagg + 4 * SM;                                 // [sumK][DL] local features
   float4* sdem = reinterpret_cast<float4*>(sx + (size_t)sumK * DL);  // [sumK]
-  int32_t* spop = reinterpret_cast<int32_t*>(sdem + sumK);   // [pop][N] the generation's genomes
-  int32_t* sgenes = spop + (((size_t)pop * N + 3) & ~(size_t)3);  // [SM][N] this slice's genomes
-  __shared__ float sval[32];
-  __shared__ int sidx[32];
+  int32_t* sgenes = reinterpret_cast<int32_t*>(sdem + sumK); // [SM][N] the slice's genomes
 
-  const int tid = threadIdx.x, lane = tid & 31;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const bool unit = tid < N * H;
-  const int m = unit ? tid / H : 0, j = unit ? tid % H : 0;
-  // this thread's weights: rows j of W1 and W2 of model m, and its layer-3 column
+  const int m = unit ? tid / H : 0;
+  const int j = tid % H;
+  const int wq = j >> 5;              // warp of the model
+  // this thread's weights: rows j of W1 and W2, the layer-3 weights of unit j
   float w1[DIN], w2[H];
   float b1 = 0.f, b2 = 0.f, w3t = 0.f, w3l = 0.f;
+  int unit_off = 0;
   if (unit) {
     const float* w = P.w32 + (size_t)m * P.per_model;
 #pragma unroll
@@ -314,217 +475,311 @@ k_ga_persist(const Params P, const GaArgs g, const GaPersist G) {
     const float* W3 = W2 + H * H + H;
     w3t = __ldg(W3 + j);
     w3l = __ldg(W3 + H + j);
+    unit_off = pick(P.off, m);
   }
-  for (int e = tid; e < N; e += blockDim.x) {
-    const float* b3 = P.w32 + (size_t)e * P.per_model + H * DIN + H + H * H + H + 2 * H;
-    sb3[2 * e] = b3[0];
-    sb3[2 * e + 1] = b3[1];
+  // per-lane constants of model `lane`
+  float my_w = 0.f, my_sla = 0.f, my_b3t = 0.f, my_b3l = 0.f;
+  int my_off = 0, my_K = 1;
+  if (lane < N) {
+    const float* b3 = P.w32 + (size_t)lane * P.per_model + H * DIN + H + H * H + H + 2 * H;
+    my_b3t = __ldg(b3);
+    my_b3l = __ldg(b3 + 1);
+    my_w = pick(P.w, lane);
+    my_sla = pick(P.sla, lane);
+    my_off = pick(P.off, lane);
+    my_K = pick(P.K, lane);
   }
+  for (int e = tid; e < N * SM * H; e += blockDim.x) sh1[e] = 0.f;
   for (int e = tid; e < sumK * DL; e += blockDim.x) sx[e] = P.x[e];
   for (int e = tid; e < sumK; e += blockDim.x) sdem[e] = P.dem[e];
+  if (tid == 0) s_abort = 0;
+  __syncthreads();
+
   const uint64_t sd = *G.seed;
-  const int c0 = blockIdx.x * G.slice;
-  const int c1 = min(pop, c0 + G.slice);
-  const int ns = c1 - c0;
-  for (int e = tid; e < ns * N; e += blockDim.x) {  // initial population of this slice
-    const int c = c0 + e / N, i = e % N;
-    const int gene = ga_unif(ga_rng(sd, 0, (uint32_t)c, kGaInit, (uint32_t)i), (uint32_t)g.K[i]);
-    G.pop0[(size_t)c * N + i] = gene;
-    sgenes[e] = gene;
+  const int c0 = blockIdx.x * SM;
+  const int ns = min(SM, pop - c0);
+  const float nz = (float)N * P.agg_scale[3];
+  const bool child_warp = warp < ns;
+  const int last_warp = (int)(blockDim.x >> 5) - 1;  // never a child warp (blockDim > 32 * SM)
+  const uint32_t cg = (uint32_t)(c0 + warp);  // the child slot of a child warp
+  auto fail = [&]() {
+    atomicOr(P.status, kStatusTimeout);
+    s_abort = 1;
+  };
+
+  // a child's genes are in place (lane i holds gene i): record it (shared memory and
+  // the ring slot of its generation, tag `tag`) and its aggregate state
+  auto place = [&](int gene, GaRec* ring_slot, uint32_t tag) {
+    float a0 = 0.f, a1 = 0.f, a2 = 0.f;
+    if (lane < N) {
+      sgenes[warp * N + lane] = gene;
+      const float4 d = sdem[my_off + gene];
+      a0 = d.x; a1 = d.y; a2 = d.z;
+    }
+    const uint32_t byte = lane < N ? (uint32_t)gene : 0u;
+    const uint32_t lo = __reduce_or_sync(0xffffffffu, lane < 4 ? byte << (8 * lane) : 0u);
+    const uint32_t hi = __reduce_or_sync(0xffffffffu, lane >= 4 && lane < 8 ? byte << (8 * (lane - 4)) : 0u);
+    if (lane == 0) { s_glo[warp] = lo; st_word(&ring_slot[cg].glo, tagged(tag, lo)); }
+    if (lane == 1) { s_ghi[warp] = hi; st_word(&ring_slot[cg].ghi, tagged(tag, hi)); }
+#pragma unroll
+    for (int o = 4; o > 0; o >>= 1) {  // lanes 0-7 hold the models
+      a0 += __shfl_xor_sync(0xffffffffu, a0, o);
+      a1 += __shfl_xor_sync(0xffffffffu, a1, o);
+      a2 += __shfl_xor_sync(0xffffffffu, a2, o);
+    }
+    if (lane == 0) {
+      sagg[4 * warp + 0] = a0 * P.agg_scale[0];
+      sagg[4 * warp + 1] = a1 * P.agg_scale[1];
+      sagg[4 * warp + 2] = a2 * P.agg_scale[2];
+      sagg[4 * warp + 3] = a1;  // raw VRAM sum for the constraint
+    }
+  };
+  if (child_warp) {  // initial population (generation 0, tag 1)
+    const int gene = lane < N ? ga_unif(ga_rng(sd, 0, cg, kGaInit, (uint32_t)lane), (uint32_t)my_K) : 0;
+    place(gene, G.rec, 1u);
   }
   __syncthreads();
-  const float nz = (float)N * P.agg_scale[3];
 
   for (int gen = 0; gen < G.gens; ++gen) {
-    int32_t* cur = (gen & 1) ? G.pop1 : G.pop0;
-    int32_t* nxt = (gen & 1) ? G.pop0 : G.pop1;
-    float* fit = (gen & 1) ? G.fit1 : G.fit0;
-    // ---- aggregate state of every individual of the slice ----
-    if (tid < ns) {
-      float A0 = 0.f, A1 = 0.f, A2 = 0.f;
-      for (int i = 0; i < N; ++i) {
-        const float4 d = sdem[P.off[i] + sgenes[tid * N + i]];
-        A0 += d.x; A1 += d.y; A2 += d.z;
-      }
-      sagg[4 * tid + 0] = A0 * P.agg_scale[0];
-      sagg[4 * tid + 1] = A1 * P.agg_scale[1];
-      sagg[4 * tid + 2] = A2 * P.agg_scale[2];
-      sagg[4 * tid + 3] = A1;  // raw VRAM sum for the constraint
+    const uint32_t tag = (uint32_t)gen + 1u;
+    const int slot = gen % G.ring;
+    GaRec* rec_cur = G.rec + (size_t)slot * pop;
+    GaRec* rec_nxt = G.rec + (size_t)((gen + 1) % G.ring) * pop;
+    GaBest* best_cur = G.best + (size_t)slot * gridDim.x;
+    const bool last = gen + 1 == G.gens;
+    // ---- the step below overwrites generation gen + 1 - ring: read every CTA's
+    // progress now, check it after the objective ----
+    const int need = gen + 2 - G.ring;
+    unsigned int pv[8] = {~0u, ~0u, ~0u, ~0u, ~0u, ~0u, ~0u, ~0u};
+    const bool lag_check = warp == last_warp && need > 0 && !last;
+    if (lag_check) {
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+        if (lane + 32 * u < (int)gridDim.x) pv[u] = ld_u32(G.prog + lane + 32 * u);
     }
-    __syncthreads();
-    // ---- layer 1: unit j of model m for every individual ----
+    // ---- layer 1 ----
     if (unit) {
 #pragma unroll
       for (int c = 0; c < SM; ++c) {
         if (c < ns) {
-          const float4* xr = reinterpret_cast<const float4*>(sx + (size_t)(P.off[m] + sgenes[c * N + m]) * DL);
-          float u0 = b1, u1 = 0.f;
-#pragma unroll
-          for (int q = 0; q < DL / 4; ++q) {
-            const float4 v = xr[q];
-            u0 = fmaf(w1[4 * q + 0], v.x, u0);
-            u1 = fmaf(w1[4 * q + 1], v.y, u1);
-            u0 = fmaf(w1[4 * q + 2], v.z, u0);
-            u1 = fmaf(w1[4 * q + 3], v.w, u1);
-          }
+          const float4* xr = reinterpret_cast<const float4*>(sx + (size_t)(unit_off + sgenes[c * N + m]) * DL);
+          const float4 v0 = xr[0], v1 = xr[1];
           const float4 a = *reinterpret_cast<const float4*>(sagg + 4 * c);
-          u0 = fmaf(w1[DL + 0], a.x, u0);
-          u1 = fmaf(w1[DL + 1], a.y, u1);
-          u0 = fmaf(w1[DL + 2], a.z, u0);
-          u1 = fmaf(w1[DL + 3], nz, u1);
+          float u0 = b1, u1 = 0.f;
+          u0 = fmaf(w1[0], v0.x, u0); u1 = fmaf(w1[1], v0.y, u1);
+          u0 = fmaf(w1[2], v0.z, u0); u1 = fmaf(w1[3], v0.w, u1);
+          u0 = fmaf(w1[4], v1.x, u0); u1 = fmaf(w1[5], v1.y, u1);
+          u0 = fmaf(w1[6], v1.z, u0); u1 = fmaf(w1[7], v1.w, u1);
+          u0 = fmaf(w1[8], a.x, u0); u1 = fmaf(w1[9], a.y, u1);
+          u0 = fmaf(w1[10], a.z, u0); u1 = fmaf(w1[11], nz, u1);
           sh1[((size_t)m * SM + c) * H + j] = relu(u0 + u1);
         }
       }
     }
     __syncthreads();
-    // ---- layers 2 and 3: unit j of model m for every individual ----
+    if (s_abort) return;
+    // ---- layers 2 and 3 (rows past the slice's end hold zeros) ----
     if (unit) {
       const float* h1 = sh1 + (size_t)m * SM * H;
-      float acc[SM];
+      // even and odd k accumulate apart, two fused multiply-adds per instruction
+      float2 acc2[SM];
 #pragma unroll
-      for (int c = 0; c < SM; ++c) acc[c] = b2;
+      for (int c = 0; c < SM; ++c) acc2[c] = make_float2(b2, 0.f);
 #pragma unroll
-      for (int k = 0; k < H; k += 4) {
+      for (int p = 0; p < H / 4; ++p) {
+        const float2 wa = make_float2(w2[4 * p + 0], w2[4 * p + 1]);
+        const float2 wb = make_float2(w2[4 * p + 2], w2[4 * p + 3]);
 #pragma unroll
         for (int c = 0; c < SM; ++c) {
-          if (c < ns) {
-            const float4 hk = *reinterpret_cast<const float4*>(h1 + c * H + k);
-            acc[c] = fmaf(w2[k + 0], hk.x, acc[c]);
-            acc[c] = fmaf(w2[k + 1], hk.y, acc[c]);
-            acc[c] = fmaf(w2[k + 2], hk.z, acc[c]);
-            acc[c] = fmaf(w2[k + 3], hk.w, acc[c]);
-          }
+          const float4 hk = *reinterpret_cast<const float4*>(h1 + c * H + 4 * p);
+          acc2[c] = fma2(wa, make_float2(hk.x, hk.y), acc2[c]);
+          acc2[c] = fma2(wb, make_float2(hk.z, hk.w), acc2[c]);
         }
       }
-      const int hh = j >> 5;  // which warp of the model's 64 units
+      float v[2 * SM];
 #pragma unroll
       for (int c = 0; c < SM; ++c) {
-        if (c < ns) {
-          const float h2 = relu(acc[c]);
-          float tt = w3t * h2, ll = w3l * h2;
+        const float h2 = relu(acc2[c].x + acc2[c].y);
+        v[c] = w3t * h2;
+        v[SM + c] = w3l * h2;
+      }
+      fold<8>(v, 0);
+      fold<4>(v, 1);
+      fold<2>(v, 2);
+      fold<1>(v, 3);
+      const float out = v[0] + __shfl_xor_sync(0xffffffffu, v[0], 16);
+      // value index 8 * bit0 + 4 * bit1 + 2 * bit2 + bit3: bit0 thr / lat, the rest the candidate
+      const int kind = lane & 1;
+      const int c = 4 * ((lane >> 1) & 1) + 2 * ((lane >> 2) & 1) + ((lane >> 3) & 1);
+      if (lane < 16) spart[((wq * SM + c) * N + m) * 2 + kind] = out;
+    }
+    __syncthreads();
+    // ---- objective and constraints: warp c, lane i = model i ----
+    if (child_warp) {
+      float J = 0.f, pen = 0.f;
+      bool ok = true;
+      if (lane < N) {
+        float t = my_b3t, l = my_b3l;
 #pragma unroll
-          for (int o = 16; o > 0; o >>= 1) {
-            tt += __shfl_xor_sync(0xffffffffu, tt, o);
-            ll += __shfl_xor_sync(0xffffffffu, ll, o);
-          }
-          if (lane == 0) {
-            spart[((hh * SM + c) * N + m) * 2 + 0] = tt;
-            spart[((hh * SM + c) * N + m) * 2 + 1] = ll;
-          }
+        for (int w = 0; w < WPM; ++w) {
+          t += spart[((w * SM + warp) * N + lane) * 2 + 0];
+          l += spart[((w * SM + warp) * N + lane) * 2 + 1];
+        }
+        t = out_act(P, t);
+        l = out_act(P, l);
+        J = my_w * t;
+        ok = l <= my_sla;
+        const float over = l - my_sla;
+        pen = over > 0.f ? over : 0.f;
+      }
+#pragma unroll
+      for (int o = 4; o > 0; o >>= 1) {  // lanes 0-7 hold the models
+        J += __shfl_xor_sync(0xffffffffu, J, o);
+        pen += __shfl_xor_sync(0xffffffffu, pen, o);
+      }
+      ok = __all_sync(0xffffffffu, ok);
+      if (lane == 0) {
+        bool feas = sagg[4 * warp + 3] <= P.vram_cap;
+        if (P.objective == MF_OBJ_WEIGHTED_THR) feas = feas && ok;
+        else J = fmaf(-P.soft_penalty, pen, J);
+        if (J != J) feas = false;
+        const float f = feas ? J : -INFINITY;
+        st_word(&rec_cur[cg].fw, tagged(tag, __float_as_uint(f)));
+        s_fit[warp] = f;
+      }
+    }
+    if (lag_check) {
+      bool ok = false;
+      for (uint32_t n = 0; n < kGaSpinLimit; ++n) {
+        bool mine = true;
+#pragma unroll
+        for (int u = 0; u < 8; ++u) mine = mine && pv[u] >= (unsigned int)need;
+        if (__all_sync(0xffffffffu, mine)) { ok = true; break; }
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          if (lane + 32 * u < (int)gridDim.x) pv[u] = ld_u32(G.prog + lane + 32 * u);
+      }
+      if (!ok && lane == 0) fail();
+    }
+    __syncthreads();
+    if (s_abort) return;
+    // ---- the last warp publishes the slice's fittest individual ----
+    if (warp == last_warp) {
+      float f = lane < ns ? s_fit[lane] : -INFINITY;
+      int s = lane < ns ? c0 + lane : -1;
+      warp_best(f, s);
+      if (lane == 0) {
+        GaBest* b = best_cur + blockIdx.x;
+        st_word(&b->glo, tagged(tag, s_glo[s - c0]));
+        st_word(&b->ghi, tagged(tag, s_ghi[s - c0]));
+        st_word(&b->sw, tagged(tag, (uint32_t)s));
+        st_word(&b->fw, tagged(tag, __float_as_uint(f)));
+      }
+    }
+    if (last) {  // CTA 0: the fittest individual of the last generation
+      if (blockIdx.x == 0 && warp == 0) {
+        float f;
+        int s;
+        uint32_t lo, hi;
+        const bool ok = best_of_ctas(best_cur, gridDim.x, tag, f, s, lo, hi);
+        if (!ok) {
+          if (lane == 0) atomicOr(P.status, kStatusTimeout);
+        } else {
+          const uint64_t g8 = (uint64_t)lo | ((uint64_t)hi << 32);
+          if (lane < N) G.out_genome[lane] = (int)((g8 >> (8 * lane)) & 0xFF);
+          if (lane == 0) *G.out_fit = f;
         }
       }
+      return;
     }
-    __syncthreads();
-    // ---- objective and constraints of the slice ----
-    if (tid < ns) {
-      Acc acc;
-      acc.init();
-      for (int i = 0; i < N; ++i) {
-        const float t = spart[((0 * SM + tid) * N + i) * 2] + spart[((1 * SM + tid) * N + i) * 2] + sb3[2 * i];
-        const float l =
-            spart[((0 * SM + tid) * N + i) * 2 + 1] + spart[((1 * SM + tid) * N + i) * 2 + 1] + sb3[2 * i + 1];
-        acc.add(P, i, out_act(P, t), out_act(P, l));
+    // ---- next generation: warp c breeds child c0 + c ----
+    if (child_warp) {
+      const uint32_t GEN = (uint32_t)gen + 1u;
+      const ChildDraws d = child_draws(g, sd, GEN, cg, lane, N, my_K);
+      uint32_t lo = 0, hi = 0;
+      bool ok = true;
+      const bool elite = g.elitism && cg == 0;
+      if (elite) {  // slot 0 keeps the fittest (lowest slot among equals), unmutated
+        float f;
+        int s;
+        ok = best_of_ctas(best_cur, gridDim.x, tag, f, s, lo, hi);
+      } else {
+        float fa = -INFINITY, fb = -INFINITY;
+        uint32_t la = 0, ha = 0, lb = 0, hb = 0;
+        if (d.ta >= 0) ok = fetch_rec(rec_cur + d.ta, tag, fa, la, ha);
+        if (ok && d.tb >= 0) ok = fetch_rec(rec_cur + d.tb, tag, fb, lb, hb);
+        ok = __all_sync(0xffffffffu, ok);
+        if (ok) ok = tournament_winner(g, sd, GEN, cg, kGaTourA, rec_cur, tag, d.ta, fa, la, ha);
+        if (ok) ok = tournament_winner(g, sd, GEN, cg, kGaTourB, rec_cur, tag, d.tb, fb, lb, hb);
+        lo = d.take_b ? lb : la;
+        hi = d.take_b ? hb : ha;
       }
-      acc.finish(P, sagg[4 * tid + 3]);
-      fit[c0 + tid] = acc.J;
-    }
-    grid_barrier(G.flags, gridDim.x, (unsigned int)gen + 1u, P.status);
-    // ---- the generation's genomes and fitness into shared memory, through L2 ----
-    {
-      const int n4 = (pop * N) >> 2;
-      const int4* src = reinterpret_cast<const int4*>(cur);
-      int4* dst = reinterpret_cast<int4*>(spop);
-      for (int e = tid; e < n4; e += blockDim.x) dst[e] = __ldcg(src + e);
-      for (int e = 4 * n4 + tid; e < pop * N; e += blockDim.x) spop[e] = __ldcg(cur + e);
-      for (int e = tid; e < pop; e += blockDim.x) sfit[e] = __ldcg(fit + e);
-    }
-    __syncthreads();
-    if (gen + 1 == G.gens) break;
-    // ---- next generation for the slice ----
-    const uint32_t GEN = (uint32_t)gen + 1u;
-    if (g.elitism && c0 == 0) {  // slot 0 keeps the fittest (lowest slot among equals)
-      const int e = block_argmax(sfit, pop, sval, sidx);
-      if (tid < N) sgenes[tid] = spop[(size_t)e * N + tid];
-    }
-    if (tid < ns && !(g.elitism && c0 + tid == 0)) {
-      const int c = c0 + tid;
-      const int a = tournament(g, sfit, sd, GEN, (uint32_t)c, kGaTourA);
-      const int b = tournament(g, sfit, sd, GEN, (uint32_t)c, kGaTourB);
-      for (int i = 0; i < N; ++i) {
-        const uint64_t rc = ga_rng(sd, GEN, (uint32_t)c, kGaCross, (uint32_t)i);
-        int gene = spop[(size_t)((rc >> 63) ? b : a) * N + i];
-        const uint64_t rm = ga_rng(sd, GEN, (uint32_t)c, kGaMut, (uint32_t)i);
-        if ((uint32_t)(rm >> 40) < g.mut_thr)
-          gene = ga_unif(ga_rng(sd, GEN, (uint32_t)c, kGaMutVal, (uint32_t)i), (uint32_t)g.K[i]);
-        sgenes[tid * N + i] = gene;
+      if (!ok) {
+        if (lane == 0) fail();
+      } else {
+        int gene = (int)(((lane < 4 ? lo : hi) >> (8 * (lane & 3))) & 0xFF);
+        if (!elite && d.mutate) gene = d.mval;
+        place(gene, rec_nxt, tag + 1u);
       }
     }
     __syncthreads();
-    for (int e = tid; e < ns * N; e += blockDim.x) nxt[(size_t)c0 * N + e] = sgenes[e];
-    __syncthreads();
+    if (s_abort) return;
+    if (tid == 0) st_u32(G.prog + blockIdx.x, (unsigned int)gen + 1u);  // generation gen fully read
   }
-  // fittest individual of the last population
-  if (blockIdx.x == 0) {
-    const int e = block_argmax(sfit, pop, sval, sidx);
-    if (tid < N) G.out_genome[tid] = spop[(size_t)e * N + tid];
-    if (tid == 0) *G.out_fit = sfit[e];
-  }
-}
-
-size_t ga_persist_smem(int N, int sumK, int pop) {
-  const size_t floats = (size_t)N * kGaMaxSlice * 64 + 4 * kGaMaxSlice * (size_t)N + 4 * kGaMaxSlice +
-                        2 * MF_MAX_MODELS + (size_t)((pop + 3) & ~3) + (size_t)sumK * 8;
-  return floats * sizeof(float) + sizeof(float4) * (size_t)sumK +
-         sizeof(int32_t) * ((((size_t)pop * N + 3) & ~(size_t)3) + (size_t)kGaMaxSlice * N);
 }
 
 mf_status ga_run_persistent(mf_ctx* c, const mf_ga_params* g, uint64_t seed, cudaStream_t s) {
   const Params& P = c->P;
   const int N = P.n_models;
-  if (!(P.d_local == 8 && P.h1 == 64 && P.h2 == 64 && N * 64 <= 512)) return MF_EUNSUPPORTED;
+  if (!(P.d_local == 8 && P.h1 == 64 && P.h2 == 64 && N <= 8)) return MF_EUNSUPPORTED;
   const int pop = g->pop;
-  int slice = (pop + c->num_sms - 1) / c->num_sms;
-  if (slice < 1) slice = 1;
-  if (slice > kGaMaxSlice) return MF_EUNSUPPORTED;
-  const int ctas = (pop + slice - 1) / slice;
-  const int threads = ((N * 64 > 256 ? N * 64 : 256) + 31) / 32 * 32;
+  const int ctas = (pop + kGaMaxSlice - 1) / kGaMaxSlice;
+  if (ctas > 256) return MF_EUNSUPPORTED;  // progress counters: eight per lane of one warp
+  // one thread per (model, hidden unit), at least one warp past the 8 child warps;
+  // register budgets of 384 (up to six models) and 512 threads
+  const int threads = std::max(N * 64, 32 * (kGaMaxSlice + 1));
+  const void* fn = threads <= 384 ? (const void*)k_ga_persist<384> : (const void*)k_ga_persist<512>;
   const int sumK = P.off[N - 1] + P.K[N - 1];
-  const size_t smem = ga_persist_smem(N, sumK, pop);
+  const size_t smem = sizeof(float) * ((size_t)N * kGaMaxSlice * 64 + (size_t)4 * kGaMaxSlice * N +
+                                       4 * kGaMaxSlice + (size_t)sumK * 8) +
+                      sizeof(float4) * (size_t)sumK + sizeof(int32_t) * (size_t)kGaMaxSlice * N;
   if (smem > 200 * 1024) return MF_EUNSUPPORTED;
-  // two register budgets: up to 384 threads (N <= 6) and up to 512 (N <= 8)
-  const void* fn = threads <= 384 ? (const void*)k_ga_persist<8, 384> : (const void*)k_ga_persist<8, 512>;
   MF_CUDA(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024));
   int per_sm = 0;
   MF_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, threads, smem));
   if (per_sm * c->num_sms < ctas) return MF_EUNSUPPORTED;
-  if (pop > c->ga_cap) {
+  // scratch: records [ring][pop], CTA bests [ring][ctas], progress [ctas]
+  const int ring = std::min(g->gens + 1, kGaRingMax);
+  const size_t recb = sizeof(GaRec) * ring * (size_t)pop, bestb = sizeof(GaBest) * ring * (size_t)ctas;
+  const size_t need = recb + bestb + sizeof(unsigned int) * (size_t)ctas;
+  if (need > c->gap_bytes) {
     MF_CUDA(cudaStreamSynchronize(s));
-    cudaFree(c->d_pop[0]); cudaFree(c->d_pop[1]); cudaFree(c->d_fit); cudaFree(c->d_pred);
-    c->d_pop[0] = c->d_pop[1] = nullptr; c->d_fit = c->d_pred = nullptr;
-    c->ga_cap = 0;
-    MF_CUDA(cudaMalloc(&c->d_pop[0], sizeof(int32_t) * (size_t)pop * N));
-    MF_CUDA(cudaMalloc(&c->d_pop[1], sizeof(int32_t) * (size_t)pop * N));
-    MF_CUDA(cudaMalloc(&c->d_fit, sizeof(float) * (size_t)pop));
-    MF_CUDA(cudaMalloc(&c->d_pred, sizeof(float) * 2 * (size_t)pop * N));
-    c->ga_cap = pop;
-    if (c->ga_exec) { cudaGraphExecDestroy(c->ga_exec); c->ga_exec = nullptr; }
+    cudaFree(c->d_gap);
+    c->d_gap = nullptr;
+    c->gap_bytes = 0;
+    MF_CUDA(cudaMalloc(&c->d_gap, need));
+    c->gap_bytes = need;
   }
   if (!c->d_ga_out) MF_CUDA(cudaMalloc(&c->d_ga_out, 128));
   mf_status st = ensure_host_stage(c, 256);
   if (st != MF_OK) return st;
-  int32_t* out_genome = (int32_t*)c->d_ga_out;
-  float* out_fit = (float*)(out_genome + N);
+  char* base = (char*)c->d_gap;
+  GaPersist G{};
+  G.rec = (GaRec*)base;
+  G.best = (GaBest*)(base + recb);
+  G.prog = (unsigned int*)(base + recb + bestb);
+  G.out_genome = (int32_t*)c->d_ga_out;
+  G.out_fit = (float*)(G.out_genome + N);
   uint64_t* d_seed = (uint64_t*)((char*)c->d_ga_out + 64);
-  // the odd generations' fitness and the per-CTA barrier flags live in the per-model
-  // output buffer (2 * pop * N words >= pop + ctas)
-  float* fit1 = c->d_pred;
-  unsigned int* flags = reinterpret_cast<unsigned int*>(c->d_pred + pop);
+  G.seed = d_seed;
+  G.gens = g->gens;
+  G.ring = ring;
   uint64_t* h_seed = (uint64_t*)((char*)c->h_stage + 128);
   *h_seed = seed;
   MF_CUDA(cudaMemcpyAsync(d_seed, h_seed, sizeof(uint64_t), cudaMemcpyHostToDevice, s));
-  MF_CUDA(cudaMemsetAsync(flags, 0, sizeof(unsigned int) * (size_t)ctas, s));
+  // tags of a previous run must not match: clear the records, bests and counters
+  MF_CUDA(cudaMemsetAsync(c->d_gap, 0, need, s));
   GaArgs a = make_args(c, g);
-  GaPersist G{c->d_pop[0], c->d_pop[1], c->d_fit, fit1, flags, out_genome, out_fit, d_seed, g->gens, slice};
   Params Pc = P;
   void* args[] = {(void*)&Pc, (void*)&a, (void*)&G};
   MF_CUDA(cudaLaunchCooperativeKernel(fn, dim3(ctas), dim3(threads), args, smem, s));

@@ -76,6 +76,7 @@ static void free_ctx(mf_ctx* c) {
   cudaFree(c->d_fit);
   cudaFree(c->d_pred);
   cudaFree(c->d_ga_out);
+  cudaFree(c->d_gap);
   if (c->ga_exec) cudaGraphExecDestroy(c->ga_exec);
   if (c->cap_stream) cudaStreamDestroy(c->cap_stream);
   for (int j = 0; j < 3; ++j)

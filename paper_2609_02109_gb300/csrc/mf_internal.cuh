@@ -200,6 +200,8 @@ struct mf_ctx {
   float* d_fit = nullptr;
   float* d_pred = nullptr;
   void* d_ga_out = nullptr;       // best genome [N] int32, then its fitness (float), then the seed (u64)
+  void* d_gap = nullptr;          // cooperative GA kernel: byte genomes, fitness, barrier flags, CTA bests
+  size_t gap_bytes = 0;
   int ga_cap = 0;
   cudaStream_t cap_stream = nullptr;
   cudaGraphExec_t ga_exec = nullptr;

@@ -49,7 +49,8 @@ CASES = {
     "one_model": ([200], 8, 9.0, "weighted_thr", dict(W.GA_PARAMS, pop=50, gens=25, mutation_p=0.2)),
     "pop_two_one_gen": ([6, 7, 8], 9, 20.0, "weighted_thr", dict(W.GA_PARAMS, pop=2, gens=1)),
     "single_generation": ([12, 9, 9, 9, 9], 5, 30.0, "weighted_thr", dict(W.GA_PARAMS, gens=1)),
-    "graph_fallback_pop_over_8_per_sm": ([6, 7, 8], 9, 20.0, "weighted_thr",
+    # eight models take a whole SM per CTA: a population above 8 per SM cannot be resident
+    "graph_fallback_pop_over_8_per_sm": ([5] * 8, 7, 45.0, "weighted_thr",
                                          dict(W.GA_PARAMS, pop=9 * 160, gens=12)),
 }
 
@@ -65,7 +66,8 @@ def test_ga_run_reproduces_oracle_run_exactly(mf, oracle_mod, name):
     prob = _problem(name)
     g = CASES[name][4]
     o = oracle_mod.Oracle(prob)
-    persistent = -(-g["pop"] // _sms()) <= MAX_SLICE
+    persistent = not name.startswith("graph_fallback")
+    assert persistent or -(-g["pop"] // _sms()) > MAX_SLICE
     with mf.Context(prob) as ctx:
         for seed in (1000, 1001, 2 ** 40 + 3):
             J, genome = ctx.ga_run(g, seed)
