@@ -228,3 +228,18 @@ def test_ga_run_reports_oracle_score_of_its_genome(mf, oracle_mod):
             Jo, f, pred, _ = o.score_digits(genome)
             assert f and abs(J - Jo) <= 1e-5 * max(abs(Jo), float(np.abs(pred[:, 0]) @ prob["obj_w"]))
             assert 0 <= genome.min() and all(genome < prob["n_options"])
+
+
+@pytest.mark.parametrize("world", [2, 3, 7])
+def test_index_range_shards_merge_to_the_full_search(mf, world):
+    """The multi-GPU split run rank by rank on one GPU: every shard's range search,
+    merged by the exchange step's merge, equals the single search of the space."""
+    from paper_2609_02109_gb300 import shard
+    prob = PROBLEMS["tight"]
+    with mf.Context(prob) as ctx:
+        full = ctx.search(32)
+        parts = [ctx.search(32, *shard.shard_range(ctx.space_size, r, world)) for r in range(world)]
+    m = shard.merge_results(parts, 32)
+    assert m["count"] == full["count"] and m["best_idx"] == full["best_idx"]
+    assert np.array_equal(m["topk_idx"], full["topk_idx"])
+    assert np.array_equal(m["topk_score"], full["topk_score"])
