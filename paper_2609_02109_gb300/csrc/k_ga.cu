@@ -267,16 +267,6 @@ struct GaPersist {
   int ring;
 };
 
-// fma.rn.f32x2: two fp32 fused multiply-adds (each rounded as fmaf) in one instruction.
-__device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
-  unsigned long long r;
-  asm("fma.rn.f32x2 %0, %1, %2, %3;"
-      : "=l"(r)
-      : "l"(*reinterpret_cast<unsigned long long*>(&a)), "l"(*reinterpret_cast<unsigned long long*>(&b)),
-        "l"(*reinterpret_cast<unsigned long long*>(&c)));
-  return *reinterpret_cast<float2*>(&r);
-}
-
 __device__ __forceinline__ unsigned long long ld_word(const unsigned long long* p) {
   unsigned long long v;
   asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
@@ -422,16 +412,6 @@ __device__ __forceinline__ bool tournament_winner(const GaArgs& g, uint64_t sd, 
   lo = __shfl_sync(0xffffffffu, lo, src);
   hi = __shfl_sync(0xffffffffu, hi, src);
   return ok;
-}
-
-// a[i] for a per-model array of the kernel parameters, read with constant indices
-// (a runtime index into a parameter array would copy it to local memory)
-template <typename T>
-__device__ __forceinline__ T pick(const T (&a)[MF_MAX_MODELS], int i) {
-  T v = a[0];
-#pragma unroll
-  for (int k = 1; k < MF_MAX_MODELS; ++k) v = k == i ? a[k] : v;
-  return v;
 }
 
 template <int MAXT>

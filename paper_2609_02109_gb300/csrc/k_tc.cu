@@ -8,7 +8,8 @@
 //   layer 2   D2[128 x h2]  = H1[128 x h1] . W2^T    (+ b2, ReLU in the epilogue)
 //   layer 3   D3[128 x n3] += H2[128 x h2] . B3_i^T  B3_i puts W3_i's two rows in
 //                                                    columns i (thr) and n3/2 + i (lat),
-//                                                    so D3 accumulates all N models.
+//                                                    so D3 accumulates all N models
+//                                                    (b3 is added in the final epilogue).
 //
 // One persistent CTA per SM runs up to four independent 128-row pipelines of
 // four warps each (warp q of a pipeline owns TMEM lanes 32q..32q+31).  Each
@@ -20,10 +21,11 @@
 // that the pipeline's threads wait on (bounded; a wait that gives up raises the
 // status word and the kernel runs to completion without further waits).
 //
-// Biases ride in the MMAs: b1 in A1's constant-1 column; b2 and b3 through a
-// constant block of ones that sits in tensor memory right after each layer's
-// activations (one extra K = 16 step whose B rows hold the bias as a bf16 hi/lo
-// pair), so the epilogues are only load -> ReLU + round -> store.  The
+// b1 rides in A1's constant-1 column and b2 in a constant block of ones that sits
+// in tensor memory right after H1 (one extra K = 16 step whose B rows hold the bias
+// as a bf16 hi/lo pair), so the hidden epilogues are only load -> ReLU + round ->
+// store.  b3 is added in fp32 in the final epilogue: a bias step of layer 3 would
+// cost a whole MMA issue (~60 cycles of the issuing thread) for two numbers.  The
 // aggregate enters layer 1 as a bf16 hi/lo pair as well (two columns per
 // component with the same weight), so its rounding error is ~2^-16, not 2^-9.
 //
@@ -214,7 +216,13 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   extern __shared__ __align__(1024) unsigned char smem[];
   __shared__ uint32_t s_tmem;
   __shared__ int s_abort;
+  __shared__ float s_b3[MF_MAX_MODELS][2];
   const int tid = threadIdx.x;
+  // compile-time K-step counts must be the layout's (else no MMA may run)
+  if ((S1 > 0 && S1 != T.k1 / 16) || (S2 > 0 && S2 != T.h1 / 16 + 1) || (S3 > 0 && S3 != T.hl / 16)) {
+    if (tid == 0) atomicOr(P.status, kStatusBadInput);
+    return;
+  }
   const int warp = tid >> 5, lane = tid & 31;
   const int pipe = warp >> 2, wq = warp & 3;
   const int row = wq * 32 + lane;
@@ -253,7 +261,11 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   if (tid < N) {
     desc_s[3 * tid + 0] = smem_desc(smem_base + T.off_b1[tid], 128u, (uint32_t)(T.k1 / 8) * 128u);
     desc_s[3 * tid + 1] = smem_desc(smem_base + T.off_b2[tid], 128u, (uint32_t)((T.h1 + 16) / 8) * 128u);
-    desc_s[3 * tid + 2] = smem_desc(smem_base + T.off_b3[tid], 128u, (uint32_t)((T.hl + 16) / 8) * 128u);
+    desc_s[3 * tid + 2] = smem_desc(smem_base + T.off_b3[tid], 128u, (uint32_t)(T.hl / 8) * 128u);
+    const float* b3 = P.w32 + (size_t)tid * P.per_model + (size_t)T.h1 * P.d_in + T.h1 +
+                      (T.h2 > 0 ? (size_t)T.h2 * T.h1 + T.h2 : 0) + 2 * (size_t)T.hl;
+    s_b3[tid][0] = b3[0];
+    s_b3[tid][1] = b3[1];
   }
   // option tables with ordinary loads
   const int sumK = P.off[N - 1] + P.K[N - 1];
@@ -295,12 +307,13 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   const uint32_t tD = tp + T.col_d, tA = tp + T.col_a, tD3 = tp + T.col_d3, tOnes = tp + T.col_ones;
   const uint32_t tH1 = tOnes - (uint32_t)(T.h1 / 2);                        // layer-2 A operand
   const uint32_t tH2 = T.h2 > 0 ? tOnes - (uint32_t)(T.h2 / 2) : tH1;       // layer-3 A operand
-  const bool leader = (wq == 0 && lane == 0);
+  // the issuing thread of pipeline p sits in warp 4p + p, so the four issuers use four schedulers
+  const bool leader = (wq == (pipe & 3) && lane == 0);
   uint64_t* mbar = &bars[1 + pipe];
   uint32_t phase = 0;
   const int barid = 1 + pipe;
   const uint32_t id1 = idesc_bf16(T.h1), id2 = idesc_bf16(T.h2), id3 = idesc_bf16(T.n3);
-  const int s1 = T.k1 / 16, s2 = T.h1 / 16 + 1, s3 = T.hl / 16 + 1;
+  const int s1 = T.k1 / 16, s2 = T.h1 / 16 + 1, s3 = T.hl / 16;
   const float vcap = P.vram_cap;
 
   {  // constant ones block: word 0 = (1, 1) feeds the bias hi/lo rows of B2 and B3
@@ -475,8 +488,8 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
       if (i >= N) break;
-      const float thr = out_act(P, __uint_as_float(d3[i]));
-      const float lat = out_act(P, __uint_as_float(half3 == 8 ? d3[(8 + i) & 31] : d3[(16 + i) & 31]));
+      const float thr = out_act(P, __uint_as_float(d3[i]) + s_b3[i][0]);
+      const float lat = out_act(P, __uint_as_float(half3 == 8 ? d3[(8 + i) & 31] : d3[(16 + i) & 31]) + s_b3[i][1]);
       if (MODE == kTcList && valid && L.pred) {
         L.pred[(t * N + i) * 2 + 0] = thr;
         L.pred[(t * N + i) * 2 + 1] = lat;
@@ -571,7 +584,7 @@ size_t topk_bytes_pipe(int kcap) { return (sizeof(uint64_t) + sizeof(float)) * (
 
 size_t image_bytes(const Params& P, int k1, int n3) {
   const int hl = P.h2 > 0 ? P.h2 : P.h1;
-  const size_t per = (size_t)P.h1 * k1 * 2 + (size_t)P.h2 * (P.h1 + 16) * 2 + (size_t)n3 * (hl + 16) * 2;
+  const size_t per = (size_t)P.h1 * k1 * 2 + (size_t)P.h2 * (P.h1 + 16) * 2 + (size_t)n3 * hl * 2;
   return per * P.n_models;
 }
 
@@ -598,8 +611,9 @@ using TcFn = void (*)(const Params, const TcArgs, const RangeArgs, const TcList)
 // counts fixed at compile time, and a run-time fallback per A1 row width.
 template <int MODE>
 TcFn tc_kernel_mode(const TcArgs& T) {
-  if (T.kw == 8 && T.dle == 8 && T.h1 == 64 && T.h2 == 64) return k_score_tc<MODE, 8, 4, 1, 5, 5>;
-  if (T.kw == 16 && T.dle == 16 && T.h1 == 128 && T.h2 == 128) return k_score_tc<MODE, 16, 8, 2, 9, 9>;
+  // S1 = k1 / 16, S2 = h1 / 16 + 1 (the b2 step), S3 = hl / 16
+  if (T.kw == 8 && T.dle == 8 && T.h1 == 64 && T.h2 == 64) return k_score_tc<MODE, 8, 4, 1, 5, 4>;
+  if (T.kw == 16 && T.dle == 16 && T.h1 == 128 && T.h2 == 128) return k_score_tc<MODE, 16, 8, 2, 9, 8>;
   if (T.kw == 8) return k_score_tc<MODE, 8, -1, 0, 0, 0>;
   return k_score_tc<MODE, 16, -1, 0, 0, 0>;
 }
@@ -652,8 +666,8 @@ mf_status tc_prepare(mf_ctx* c) {
   T.pipes = 512 / T.pipe_stride;
   if (T.pipes > kTcMaxPipes) T.pipes = kTcMaxPipes;
 
-  // B operand images (K-major): B1 [h1 x k1], B2 [h2 x (h1 + 16)], B3 [n3 x (hl + 16)]
-  const int k2 = h1 + 16, k3 = hl + 16;
+  // B operand images (K-major): B1 [h1 x k1], B2 [h2 x (h1 + 16)], B3 [n3 x hl]
+  const int k2 = h1 + 16, k3 = hl;
   const size_t b1_bytes = (size_t)h1 * T.k1 * 2, b2_bytes = (size_t)h2 * k2 * 2, b3_bytes = (size_t)T.n3 * k3 * 2;
   std::vector<unsigned char> img;
   const double s3 = P.agg_scale[3];
@@ -677,7 +691,6 @@ mf_status tc_prepare(mf_ctx* c) {
     const float* W2 = b1 + h1;
     const float* b2 = W2 + (size_t)h2 * h1;
     const float* W3 = h2 > 0 ? b2 + h2 : W2;
-    const float* b3 = W3 + 2 * (size_t)hl;
     T.off_b1[i] = (uint32_t)img.size();
     img.resize(img.size() + b1_bytes, 0);
     for (int j = 0; j < h1; ++j) {
@@ -702,8 +715,6 @@ mf_status tc_prepare(mf_ctx* c) {
       put(T.off_b3[i], i, k, k3, W3[k]);
       put(T.off_b3[i], T.n3 / 2 + i, k, k3, W3[hl + k]);
     }
-    put_bias(T.off_b3[i], i, hl, k3, b3[0]);
-    put_bias(T.off_b3[i], T.n3 / 2 + i, hl, k3, b3[1]);
   }
   img.resize(round_up((int)img.size(), 16), 0);
   T.img_bytes = (uint32_t)img.size();
