@@ -129,17 +129,18 @@ class ClockSampler:
 # ---------------------------------------------------------------------------
 # CPU baseline: the oracle on a bounded sample of the same workload
 # ---------------------------------------------------------------------------
-def cpu_baseline(prob, target_s=12.0):
+def cpu_baseline(prob, target_s=15.0):
     from oracle.oracle import Oracle
     cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
     o = Oracle(prob, nthreads=cores)
-    t = time.perf_counter()
-    o.exhaustive(K_TOP, lo=0, hi=20000)
-    rate = 20000 / max(time.perf_counter() - t, 1e-6)
-    n = int(min(max(rate * target_s, 1e5), 5e7))
-    t = time.perf_counter()
-    o.exhaustive(K_TOP, lo=0, hi=n)
-    dt = time.perf_counter() - t
+    n = 200000
+    while True:  # grow the sample until it takes about target_s (at least 10 s)
+        t = time.perf_counter()
+        o.exhaustive(K_TOP, lo=0, hi=n)
+        dt = time.perf_counter() - t
+        if dt >= 10.0 or n >= 24 ** 6:
+            break
+        n = int(min(n * max(2.0, target_s / max(dt, 1e-3)), 24 ** 6))
     return {"value": n / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
             "sample": f"fp64 C oracle exhaustive search (top-32 + count) over indices [0, {n}) "
                       f"of the same N=6 space, {dt:.1f} s"}
@@ -330,7 +331,7 @@ def run_gpu(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--precision", default=os.environ.get("MF_BENCH_PRECISION", "bf16"),
