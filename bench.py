@@ -39,6 +39,23 @@ K_TOP = 32
 CHUNK = 1 << 24
 L2_FLUSH_BYTES = 256 << 20
 
+# DRAM bytes (read + write) of one scoring launch from the ncu capture summarised in
+# profiles/k_score_tc_large_n6.md, valid only while the kernel's sources are the ones
+# that were captured (sha256 prefix of k_tc.cu + mf_internal.cuh)
+NCU_TRAFFIC = {"bf16": ("064037cd705e134d", 2054144)}
+
+
+def _traffic(prec):
+    import hashlib
+    ent = NCU_TRAFFIC.get(prec)
+    if ent is None:
+        return None
+    h = hashlib.sha256()
+    for f in ("k_tc.cu", "mf_internal.cuh"):
+        with open(os.path.join(ROOT, "paper_2609_02109_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return ent[1] if h.hexdigest()[:16] == ent[0] else None
+
 
 def _peaks():
     try:
@@ -294,7 +311,7 @@ def run_gpu(args):
             roof = {"bound": "alu", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                     "frac": achieved / peak,
                     "peak_source": f"{sms} SMs x 128 FP32 lanes x 2 FLOP x {peaks.get('sm_max_mhz', 2070.0)} MHz"}
-        roof.update({"traffic": None, "kernel": "scoring kernel (one launch per 2^24 candidates)",
+        roof.update({"traffic": _traffic(prec), "kernel": "scoring kernel (one launch per 2^24 candidates)",
                      "flops_per_candidate": fpc, "launch_ms": per_launch_ms})
 
         # end to end through the C ABI from host buffers: create (uploads) + search + result
