@@ -251,17 +251,18 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   const uint32_t smem_base = smem_u32(smem);
   if (tid == 0) {
     // weights: one TMA bulk copy per 32 KB piece, all completing on bars[0]
-    mbar_arrive_expect_tx(&bars[0], T.img_bytes);
-    for (uint32_t o = 0; o < T.img_bytes; o += 32768u) {
-      const uint32_t b = T.img_bytes - o < 32768u ? T.img_bytes - o : 32768u;
-      bulk_g2s(smem + o, static_cast<const unsigned char*>(T.img) + o, b, &bars[0]);
+    mbar_arrive_expect_tx(&bars[0], T.img_copy);
+    for (uint32_t o = 0; o < T.img_copy; o += 32768u) {
+      const uint32_t b = T.img_copy - o < 32768u ? T.img_copy - o : 32768u;
+      bulk_g2s(smem + o, static_cast<const unsigned char*>(T.img) + T.img_lo + o, b, &bars[0]);
     }
   }
-  // UMMA descriptors of every model's three B operands
-  if (tid < N) {
-    desc_s[3 * tid + 0] = smem_desc(smem_base + T.off_b1[tid], 128u, (uint32_t)(T.k1 / 8) * 128u);
-    desc_s[3 * tid + 1] = smem_desc(smem_base + T.off_b2[tid], 128u, (uint32_t)((T.h1 + 16) / 8) * 128u);
-    desc_s[3 * tid + 2] = smem_desc(smem_base + T.off_b3[tid], 128u, (uint32_t)(T.hl / 8) * 128u);
+  // UMMA descriptors of the pass's models' three B operands
+  if (tid >= T.m0 && tid < T.m1) {
+    const uint32_t sb = smem_base - T.img_lo;
+    desc_s[3 * tid + 0] = smem_desc(sb + T.off_b1[tid], 128u, (uint32_t)(T.k1 / 8) * 128u);
+    desc_s[3 * tid + 1] = smem_desc(sb + T.off_b2[tid], 128u, (uint32_t)((T.h1 + 16) / 8) * 128u);
+    desc_s[3 * tid + 2] = smem_desc(sb + T.off_b3[tid], 128u, (uint32_t)(T.hl / 8) * 128u);
     const float* b3 = P.w32 + (size_t)tid * P.per_model + (size_t)T.h1 * P.d_in + T.h1 +
                       (T.h2 > 0 ? (size_t)T.h2 * T.h1 + T.h2 : 0) + 2 * (size_t)T.hl;
     s_b3[tid][0] = b3[0];
@@ -314,6 +315,7 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   const int barid = 1 + pipe;
   const uint32_t id1 = idesc_bf16(T.h1), id2 = idesc_bf16(T.h2), id3 = idesc_bf16(T.n3);
   const int s1 = T.k1 / 16, s2 = T.h1 / 16 + 1, s3 = T.hl / 16;
+  const int m0 = T.m0, m1 = T.m1;  // this pass's models
   const float vcap = P.vram_cap;
 
   {  // constant ones block: word 0 = (1, 1) feeds the bias hi/lo rows of B2 and B3
@@ -343,7 +345,7 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
 
   auto issue_mma1 = [&](int i) { mma_steps<S1>(s1, tD, tA, desc_s[3 * i + 0], id1, 0u); };
   auto issue_mma2 = [&](int i) { mma_steps<S2>(s2, tD, tH1, desc_s[3 * i + 1], id2, 0u); };
-  auto issue_mma3 = [&](int i) { mma_steps<S3>(s3, tD3, tH2, desc_s[3 * i + 2], id3, i > 0 ? 1u : 0u); };
+  auto issue_mma3 = [&](int i) { mma_steps<S3>(s3, tD3, tH2, desc_s[3 * i + 2], id3, i > m0 ? 1u : 0u); };
   // fp32 accumulators [0, width) -> ReLU -> bf16 pairs at dst
   auto epilogue = [&](int width, uint32_t dst) {
     for (int c0 = 0; c0 < width; c0 += 32) {
@@ -439,12 +441,12 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
       named_bar(barid, 128);
     };
 
-    write_a1(0);
+    write_a1(m0);
     publish();
-    for (int i = 0; i < N; ++i) {
+    for (int i = m0; i < m1; ++i) {
       if (leader) {
         tc_fence_after();
-        if (i > 0) issue_mma3(i - 1);
+        if (i > m0) issue_mma3(i - 1);
         issue_mma1(i);
         mma_commit(mbar);
       }
@@ -460,12 +462,12 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
         await_mma();
         epilogue(T.h2, tH2);  // layer 2 (bias through the ones block)
       }
-      if (i + 1 < N) write_a1(i + 1);
+      if (i + 1 < m1) write_a1(i + 1);
       publish();
     }
     if (leader) {
       tc_fence_after();
-      issue_mma3(N - 1);
+      issue_mma3(m1 - 1);
       mma_commit(mbar);
     }
     await_mma();
@@ -487,7 +489,8 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     const int half3 = T.n3 >> 1;  // thr of model i in column i, lat in column half3 + i
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
-      if (i >= N) break;
+      if (i >= m1) break;
+      if (i < m0) continue;
       const float thr = out_act(P, __uint_as_float(d3[i]) + s_b3[i][0]);
       const float lat = out_act(P, __uint_as_float(half3 == 8 ? d3[(8 + i) & 31] : d3[(16 + i) & 31]) + s_b3[i][1]);
       if (MODE == kTcList && valid && L.pred) {
@@ -501,6 +504,18 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
       sla_near = sla_near && (lat <= sla + 2e-2f * fmaxf(fabsf(sla), fabsf(lat)));
       const float over = lat - sla;
       pen += over > 0.f ? over : 0.f;
+    }
+    if (!T.pass_first && t < n) {  // the earlier passes' models
+      const float4 pr = T.partial[t];
+      J += pr.x;
+      pen += pr.y;
+      const uint32_t fl = __float_as_uint(pr.z);
+      sla_ok = sla_ok && (fl & 1u);
+      sla_near = sla_near && (fl & 2u);
+    }
+    if (!T.pass_last) {  // (uniform) hand the partial objective to the next pass
+      if (t < n) T.partial[t] = make_float4(J, pen, __uint_as_float((sla_ok ? 1u : 0u) | (sla_near ? 2u : 0u)), 0.f);
+      continue;
     }
     bool feas = valid && A1 <= vcap;
     bool cand = feas;
@@ -532,7 +547,7 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     }
   }
 
-  if (MODE == kTcRange) {
+  if (MODE == kTcRange && T.pass_last) {
     const size_t gl = ((size_t)blockIdx.x * npipes + pipe) * kcap;
     for (int e = row; e < kcap; e += 128) {
       R.lists_s[gl + e] = tk.ls[e];
@@ -604,6 +619,7 @@ void layout_smem(const Params& P, TcArgs& T, int kcap) {
 }
 
 constexpr uint32_t kSmemLimit = 227 * 1024 - 1024;  // static shared variables take the rest
+constexpr size_t kPassImageBudget = 160 * 1024;      // bf16 weights staged per pass
 
 using TcFn = void (*)(const Params, const TcArgs, const RangeArgs, const TcList);
 
@@ -625,6 +641,41 @@ constexpr uint32_t kSmemFloor = 120 * 1024;          // keeps one CTA (one TMEM 
 
 }  // namespace
 
+namespace {
+
+// Candidates per launch when the models run in several passes (the partial records of
+// one launch: 16 B each, 256 MiB).
+constexpr uint64_t kPassSpan = 1ull << 24;
+
+// Per-launch fields of pass p.
+void set_pass(TcArgs& T, int p, float4* partial) {
+  T.m0 = T.pass_m[p];
+  T.m1 = T.pass_m[p + 1];
+  T.pass_first = p == 0;
+  T.pass_last = p + 1 == T.npasses;
+  T.img_lo = T.off_b1[T.m0];
+  T.img_copy = (p + 1 < T.npasses ? T.off_b1[T.m1] : T.img_total) - T.img_lo;
+  T.partial = partial;
+}
+
+mf_status ensure_partial(mf_ctx* c, uint64_t n, cudaStream_t s, float4** out) {
+  *out = nullptr;
+  if (c->tc.npasses == 1) return MF_OK;
+  const size_t need = sizeof(float4) * (size_t)(n < kPassSpan ? (n > 0 ? n : 1) : kPassSpan);
+  if (need > c->partial_bytes) {
+    MF_CUDA(cudaStreamSynchronize(s));
+    cudaFree(c->d_partial);
+    c->d_partial = nullptr;
+    c->partial_bytes = 0;
+    MF_CUDA(cudaMalloc(&c->d_partial, need));
+    c->partial_bytes = need;
+  }
+  *out = static_cast<float4*>(c->d_partial);
+  return MF_OK;
+}
+
+}  // namespace
+
 bool tc_supported(const Params& P, std::string* why) {
   auto no = [&](const char* m) { if (why) *why = m; return false; };
   if (P.h1 % 32 || P.h1 > 256) return no("hidden1 must be a multiple of 32 up to 256");
@@ -637,7 +688,8 @@ bool tc_supported(const Params& P, std::string* why) {
   const int col_a = hmax + hmax / 2 + 8;
   const int col_d3 = round_up(col_a + k1 / 2, 16);
   if (round_up(col_d3 + n3, 32) > 512) return no("tensor-memory footprint above 512 columns");
-  if (image_bytes(P, k1, n3) > 160 * 1024) return no("bf16 weights of all models exceed the shared-memory budget");
+  if (image_bytes(P, k1, n3) / P.n_models > kPassImageBudget)
+    return no("one model's bf16 weights exceed the shared-memory budget");
   return true;
 }
 
@@ -717,7 +769,24 @@ mf_status tc_prepare(mf_ctx* c) {
     }
   }
   img.resize(round_up((int)img.size(), 16), 0);
-  T.img_bytes = (uint32_t)img.size();
+  T.img_total = (uint32_t)img.size();
+  // passes: consecutive models whose images fit the budget together
+  T.npasses = 0;
+  T.pass_m[0] = 0;
+  for (int i = 0; i < N;) {
+    int j = i + 1;
+    while (j < N && (size_t)((j + 1 < N ? T.off_b1[j + 1] : T.img_total) - T.off_b1[i]) <= kPassImageBudget) ++j;
+    T.pass_m[++T.npasses] = j;
+    i = j;
+  }
+  T.img_bytes = 0;
+  for (int p = 0; p < T.npasses; ++p) {
+    const uint32_t lo = T.off_b1[T.pass_m[p]];
+    const uint32_t hi = p + 1 < T.npasses ? T.off_b1[T.pass_m[p + 1]] : T.img_total;
+    if (hi - lo > T.img_bytes) T.img_bytes = hi - lo;
+  }
+  set_pass(T, 0, nullptr);  // single-pass defaults (a pass-0 image of all models)
+  if (T.npasses == 1) { T.pass_last = 1; }
 
   // local-feature words
   const int sumK = c->sumK;
@@ -748,7 +817,8 @@ mf_status tc_prepare(mf_ctx* c) {
   return MF_OK;
 }
 
-mf_status tc_search_chunk(mf_ctx* c, const RangeArgs& a, cudaStream_t s) {
+
+mf_status tc_search_chunk(mf_ctx* c, const RangeArgs& a, cudaStream_t s, int* nlaunch) {
   TcArgs T = c->tc;
   layout_smem(c->P, T, a.k);
   if (T.sm_total > kSmemLimit) {
@@ -764,8 +834,26 @@ mf_status tc_search_chunk(mf_ctx* c, const RangeArgs& a, cudaStream_t s) {
   }
   const uint32_t smem = T.sm_total > kSmemFloor ? T.sm_total : kSmemFloor;
   TcList L{};
-  tc_kernel(kTcRange, T)<<<c->num_sms, T.pipes * 128, smem, s>>>(c->P, T, a, L);
-  MF_CUDA(cudaGetLastError());
+  float4* partial = nullptr;
+  mf_status st = ensure_partial(c, a.len, s, &partial);
+  if (st != MF_OK) return st;
+  // one launch per pass and span of candidates; the lists and the count belong to the
+  // last pass only
+  const uint64_t span = T.npasses == 1 ? (a.len > 0 ? a.len : 1) : kPassSpan;
+  int launches = 0;
+  RangeArgs r = a;
+  for (uint64_t b = 0; b == 0 || b < a.len; b += span) {
+    r.base = a.base + b;
+    r.len = a.len - b < span ? a.len - b : span;
+    r.first = a.first && b == 0;
+    for (int p = 0; p < T.npasses; ++p) {
+      set_pass(T, p, partial);
+      tc_kernel(kTcRange, T)<<<c->num_sms, T.pipes * 128, smem, s>>>(c->P, T, r, L);
+      MF_CUDA(cudaGetLastError());
+      ++launches;
+    }
+  }
+  *nlaunch = launches;
   return MF_OK;
 }
 
@@ -775,14 +863,25 @@ mf_status tc_score_list(mf_ctx* c, const uint64_t* idx, uint64_t n, float* score
   TcArgs T = c->tc;
   layout_smem(c->P, T, 0);
   const uint32_t smem = T.sm_total > kSmemFloor ? T.sm_total : kSmemFloor;
-  const uint64_t tiles = (n + 127) / 128;
-  const uint64_t per_cta = (uint64_t)T.pipes;
-  uint64_t grid = (tiles + per_cta - 1) / per_cta;
-  if (grid > (uint64_t)c->num_sms) grid = c->num_sms;
+  float4* partial = nullptr;
+  mf_status st = ensure_partial(c, n, s, &partial);
+  if (st != MF_OK) return st;
+  const uint64_t span = T.npasses == 1 ? n : kPassSpan;
+  const int N = c->P.n_models;
   RangeArgs R{};
-  TcList L{idx, n, score, feas, pred};
-  tc_kernel(kTcList, T)<<<(unsigned)grid, T.pipes * 128, smem, s>>>(c->P, T, R, L);
-  MF_CUDA(cudaGetLastError());
+  for (uint64_t b = 0; b < n; b += span) {
+    const uint64_t m = n - b < span ? n - b : span;
+    const uint64_t tiles = (m + 127) / 128;
+    const uint64_t per_cta = (uint64_t)T.pipes;
+    uint64_t grid = (tiles + per_cta - 1) / per_cta;
+    if (grid > (uint64_t)c->num_sms) grid = c->num_sms;
+    TcList L{idx + b, m, score + b, feas ? feas + b : nullptr, pred ? pred + b * N * 2 : nullptr};
+    for (int p = 0; p < T.npasses; ++p) {
+      set_pass(T, p, partial);
+      tc_kernel(kTcList, T)<<<(unsigned)grid, T.pipes * 128, smem, s>>>(c->P, T, R, L);
+      MF_CUDA(cudaGetLastError());
+    }
+  }
   return MF_OK;
 }
 

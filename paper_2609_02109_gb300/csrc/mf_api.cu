@@ -70,6 +70,7 @@ static void free_ctx(mf_ctx* c) {
   cudaFree(c->d_wT);
   cudaFree(c->d_status);
   cudaFree(c->d_tc);
+  cudaFree(c->d_partial);
   cudaFree(c->d_scratch);
   cudaFree(c->d_pop[0]);
   cudaFree(c->d_pop[1]);
@@ -370,19 +371,21 @@ mf_status mf_search_range(mf_ctx* ctx, uint64_t lo, uint64_t hi, int32_t k, uint
     // empty range: initialise the lists through a zero-length launch of the scorer
     a.base = lo;
     a.len = 0;
-    st = tc ? tc_search_chunk(ctx, a, s) : f32_search_chunk(ctx, a, s);
+    int nl = 1;
+    st = tc ? tc_search_chunk(ctx, a, s, &nl) : f32_search_chunk(ctx, a, s);
     if (st != MF_OK) return st;
-    ++launches;
-    ++score_launches;
+    launches += nl;
+    score_launches += nl;
   }
   for (uint64_t b = lo; b < hi; b += chunk) {
     a.base = b;
     a.len = (hi - b) < chunk ? (hi - b) : chunk;
-    st = tc ? tc_search_chunk(ctx, a, s) : f32_search_chunk(ctx, a, s);
+    int nl = 1;
+    st = tc ? tc_search_chunk(ctx, a, s, &nl) : f32_search_chunk(ctx, a, s);
     if (st != MF_OK) return st;
     a.first = 0;
-    ++launches;
-    ++score_launches;
+    launches += nl;
+    score_launches += nl;
   }
   MF_CUDA(cudaEventRecord(ctx->ev[1], s));
   st = merge_lists(ctx, ls, li, grid, kcap, ts, ti, ms, mi, s);

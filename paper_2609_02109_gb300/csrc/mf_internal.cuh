@@ -46,6 +46,14 @@ struct TcArgs {
   uint32_t sm_xw, sm_dem, sm_rows, sm_desc, sm_topk, sm_bar, sm_total;  // shared-memory byte offsets
   int32_t kcap;                       // per-pipeline list length the layout was sized for
   uint32_t step[MF_MAX_MODELS];       // mixed-radix digits of the per-tile index stride (range mode)
+  // models whose weights do not fit shared memory together run in passes of consecutive
+  // models [pass_m[p], pass_m[p + 1]); each pass's image is staged on its own
+  int32_t npasses;
+  int32_t pass_m[MF_MAX_MODELS + 1];
+  // per launch: this pass's models and image bytes, and the per-candidate partial record
+  int32_t m0, m1, pass_first, pass_last;
+  uint32_t img_lo, img_copy, img_total;
+  float4* partial;                    // [candidates of the launch] (J, penalty, flags, -)
 };
 
 // Device status bits.
@@ -207,6 +215,8 @@ struct mf_ctx {
   float* d_wT = nullptr;
   uint32_t* d_status = nullptr;
   void* d_tc = nullptr;           // packed bf16 operand images (tensor-core path)
+  void* d_partial = nullptr;      // per-candidate partial objective between tensor-core passes
+  size_t partial_bytes = 0;
   size_t tc_bytes = 0;
   mf::TcArgs tc{};
   // growable scratch (search lists, merge buffers, shortlist)
@@ -283,7 +293,7 @@ mf_status select_topk(mf_ctx* c, const float* in_s, const uint64_t* in_i, int n,
 bool tc_supported(const Params& P, std::string* why);
 mf_status tc_prepare(mf_ctx* c);
 int tc_grid(const mf_ctx* c);
-mf_status tc_search_chunk(mf_ctx* c, const RangeArgs& a, cudaStream_t s);
+mf_status tc_search_chunk(mf_ctx* c, const RangeArgs& a, cudaStream_t s, int* nlaunch);
 mf_status tc_score_list(mf_ctx* c, const uint64_t* idx, uint64_t n, float* score,
                         uint8_t* feas, float* pred, cudaStream_t s);
 

@@ -38,7 +38,11 @@ def _problems():
                          sla_range=(0.3, 0.7))
     # paper's 64-32 predictor shape, eight models (16 D3 columns)
     p6432 = W.make_problem([4] * 8, 8, 64, 32, 13, 100.0, precision="bf16", sla_range=(-0.1, 0.4))
-    return {"paper": paper, "tight": tight, "stress3": stress3, "odd": odd, "p6432": p6432}
+    # five 20->128->128->2 models: 240 KB of bf16 weights, staged in two passes (3 + 2 models)
+    multipass = W.make_problem([3, 4, 2, 3, 2], 16, 128, 128, 5, 180.0, precision="bf16",
+                               sla_range=(-0.2, 0.3))
+    return {"paper": paper, "tight": tight, "stress3": stress3, "odd": odd, "p6432": p6432,
+            "multipass": multipass}
 
 
 PROBLEMS = _problems()
