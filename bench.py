@@ -203,6 +203,33 @@ def run_reference(args):
 # ---------------------------------------------------------------------------
 # GPU arm
 # ---------------------------------------------------------------------------
+def stress_throughput(mf, torch, device):
+    """The stress workload (2^32 candidates, bf16, eight 20->128->128->2 predictors in
+    three shared-memory passes), one warm-up and one timed search."""
+    prob = W.stress(precision="bf16")
+    n = 2 ** 32
+    stream = torch.cuda.current_stream(device)
+    with mf.Context(prob, device=device) as ctx:
+        ctx.search(64, chunk=1 << 26)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize(device)
+        e0.record(stream)
+        res = ctx.search(64, chunk=1 << 26)
+        e1.record(stream)
+        e1.synchronize()
+        st = ctx.stats()
+    ms = e0.elapsed_time(e1)
+    peaks, src = _peaks()
+    achieved = flops_per_candidate(prob) * n / (st["score_ms_last"] / 1e3) / 1e12
+    return {"workload": "stress exhaustive: N=8 x 16 options (2^32 joint configs), 20->128->128->2 bf16, "
+                        "soft latency penalty 0.1, VRAM cap 180 GB, top-64, chunks of 2^26",
+            "value": n / (ms / 1e3), "unit": UNIT, "ms": ms, "count": res["count"],
+            "roofline": {"achieved": achieved, "peak": float(peaks["bf16_tflops_sustained"]), "unit": "TFLOP/s",
+                         "frac": achieved / float(peaks["bf16_tflops_sustained"]),
+                         "flops_per_candidate": flops_per_candidate(prob), "peak_source": f"{src} bf16 sustained"}}
+
+
 def ga_latency(mf, torch, device, decisions_per_scenario):
     """p50/p99 of complete GA decisions (host call -> result on host) over 8 scenarios."""
     g = W.GA_PARAMS
@@ -328,6 +355,7 @@ def run_gpu(args):
                "d2h_bytes_per_step": int(st2["d2h_bytes_last"]),
                "how": "mf_create from host arrays + mf_search_exhaustive + mf_destroy, host wall clock, median"}
 
+    stress = stress_throughput(mf, torch, device) if rank == 0 and not args.no_stress else None
     ga = ga_latency(mf, torch, device, args.ga_decisions) if rank == 0 else None
     base = cpu_baseline(W.large(precision="fp32")) if (rank == 0 and world == 1 and not args.no_cpu) else None
     if rank == 0:
@@ -338,7 +366,7 @@ def run_gpu(args):
                 "cpu_baseline": base, "e2e": e2e, "gpu_launches": launches, "clocks": clk.summary(),
                 "feasible_fraction": feasible_frac, "best": {"idx": res["best_idx"], "J": res["best_score"],
                                                              "count": res["count"]},
-                "ga": ga}
+                "ga": ga, "stress": stress}
         print(json.dumps(line), flush=True)
     if dist:
         dist.barrier()
@@ -355,6 +383,7 @@ def main():
                     choices=["bf16", "fp32"])
     ap.add_argument("--ga-decisions", type=int, default=10)
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU-baseline leg")
+    ap.add_argument("--no-stress", action="store_true", help="skip the stress-workload line")
     args = ap.parse_args()
     if args.impl == "reference":
         run_reference(args)

@@ -210,7 +210,9 @@ __device__ __forceinline__ void mma_steps(int steps, uint32_t d_tmem, uint32_t a
 
 // KW: 32-bit words of an A1 row (8 or 16); AWO: word where the aggregate starts, or
 // -1 to take it from T at run time.  S1, S2, S3: K-steps of the three layers (0 = run time).
-template <int MODE, int KW, int AWO, int S1, int S2, int S3>
+// MP: the models run in several passes (T.m0..T.m1 and a partial record per candidate);
+// otherwise all N models in one launch.
+template <int MODE, int KW, int AWO, int S1, int S2, int S3, bool MP>
 __global__ void __launch_bounds__(kTcMaxPipes * 128, 1)
 k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   extern __shared__ __align__(1024) unsigned char smem[];
@@ -315,7 +317,7 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   const int barid = 1 + pipe;
   const uint32_t id1 = idesc_bf16(T.h1), id2 = idesc_bf16(T.h2), id3 = idesc_bf16(T.n3);
   const int s1 = T.k1 / 16, s2 = T.h1 / 16 + 1, s3 = T.hl / 16;
-  const int m0 = T.m0, m1 = T.m1;  // this pass's models
+  const int m0 = MP ? T.m0 : 0, m1 = MP ? T.m1 : N;  // this pass's models
   const float vcap = P.vram_cap;
 
   {  // constant ones block: word 0 = (1, 1) feeds the bias hi/lo rows of B2 and B3
@@ -505,7 +507,7 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
       const float over = lat - sla;
       pen += over > 0.f ? over : 0.f;
     }
-    if (!T.pass_first && t < n) {  // the earlier passes' models
+    if (MP && !T.pass_first && t < n) {  // the earlier passes' models
       const float4 pr = T.partial[t];
       J += pr.x;
       pen += pr.y;
@@ -513,7 +515,7 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
       sla_ok = sla_ok && (fl & 1u);
       sla_near = sla_near && (fl & 2u);
     }
-    if (!T.pass_last) {  // (uniform) hand the partial objective to the next pass
+    if (MP && !T.pass_last) {  // (uniform) hand the partial objective to the next pass
       if (t < n) T.partial[t] = make_float4(J, pen, __uint_as_float((sla_ok ? 1u : 0u) | (sla_near ? 2u : 0u)), 0.f);
       continue;
     }
@@ -547,7 +549,7 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     }
   }
 
-  if (MODE == kTcRange && T.pass_last) {
+  if (MODE == kTcRange && (!MP || T.pass_last)) {
     const size_t gl = ((size_t)blockIdx.x * npipes + pipe) * kcap;
     for (int e = row; e < kcap; e += 128) {
       R.lists_s[gl + e] = tk.ls[e];
@@ -625,17 +627,18 @@ using TcFn = void (*)(const Params, const TcArgs, const RangeArgs, const TcList)
 
 // Instantiations: the two benchmark shapes (d_L 8, 64-64 and d_L 16, 128-128) with all
 // counts fixed at compile time, and a run-time fallback per A1 row width.
-template <int MODE>
+template <int MODE, bool MP>
 TcFn tc_kernel_mode(const TcArgs& T) {
   // S1 = k1 / 16, S2 = h1 / 16 + 1 (the b2 step), S3 = hl / 16
-  if (T.kw == 8 && T.dle == 8 && T.h1 == 64 && T.h2 == 64) return k_score_tc<MODE, 8, 4, 1, 5, 4>;
-  if (T.kw == 16 && T.dle == 16 && T.h1 == 128 && T.h2 == 128) return k_score_tc<MODE, 16, 8, 2, 9, 8>;
-  if (T.kw == 8) return k_score_tc<MODE, 8, -1, 0, 0, 0>;
-  return k_score_tc<MODE, 16, -1, 0, 0, 0>;
+  if (T.kw == 8 && T.dle == 8 && T.h1 == 64 && T.h2 == 64) return k_score_tc<MODE, 8, 4, 1, 5, 4, MP>;
+  if (T.kw == 16 && T.dle == 16 && T.h1 == 128 && T.h2 == 128) return k_score_tc<MODE, 16, 8, 2, 9, 8, MP>;
+  if (T.kw == 8) return k_score_tc<MODE, 8, -1, 0, 0, 0, MP>;
+  return k_score_tc<MODE, 16, -1, 0, 0, 0, MP>;
 }
 
 TcFn tc_kernel(int mode, const TcArgs& T) {
-  return mode == kTcRange ? tc_kernel_mode<kTcRange>(T) : tc_kernel_mode<kTcList>(T);
+  if (T.npasses > 1) return mode == kTcRange ? tc_kernel_mode<kTcRange, true>(T) : tc_kernel_mode<kTcList, true>(T);
+  return mode == kTcRange ? tc_kernel_mode<kTcRange, false>(T) : tc_kernel_mode<kTcList, false>(T);
 }
 constexpr uint32_t kSmemFloor = 120 * 1024;          // keeps one CTA (one TMEM owner) per SM
 
