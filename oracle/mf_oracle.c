@@ -417,3 +417,136 @@ double orc_ga_run(const orc_problem *p, const orc_ga_params *g, uint64_t seed,
   free(fit);
   return best;
 }
+
+/* ---------------------------------------------------------------------------
+ * Fixed-context mode: Sec. III-B holds the observed state s_t fixed during the
+ * search, so each predictor g_i(lambda_i, s_t) depends on its own option only;
+ * Eq. 3 is the utility, Eq. 4 the constraints.
+ * ------------------------------------------------------------------------- */
+
+/* The observed state fed to the predictors, scaled like the aggregate. */
+static void fc_inputs(const orc_problem *p, const orc_fc *fc, double *zs) {
+  const int32_t n = p->n_models;
+  double s[4];
+  if (p->agg_scale) {
+    for (int c = 0; c < 4; ++c) s[c] = (double)p->agg_scale[c];
+  } else {
+    s[0] = 1.0 / (0.6 * n); s[1] = 1.0 / (20.0 * n); s[2] = 1.0 / (1500.0 * n); s[3] = 1.0 / 8.0;
+    for (int c = 0; c < 4; ++c) s[c] = (double)(float)s[c];
+  }
+  for (int c = 0; c < 4; ++c) zs[c] = (double)fc->obs[c] * s[c];
+}
+
+/* Model i's term of Eq. 3 for option row r: returns u and sets *fhat, *f, *ok. */
+static double fc_term(const orc_problem *p, const orc_fc *fc, int32_t i, int64_t r, const double *zs,
+                      double *fhat_out, double *f_out, int32_t *ok_out) {
+  const int32_t dl = p->d_local, din = d_in_of(p);
+  double z[din];
+  const float *x = p->local_feats + (int64_t)dl * r;
+  for (int32_t k = 0; k < dl; ++k) z[k] = (double)x[k];
+  for (int c = 0; c < 4; ++c) z[dl + c] = zs[c];
+  double fhat, lat;
+  predictor(p, i, z, &fhat, &lat, NULL);
+  /* per-variant min-max normalisation of the raw predicted throughput */
+  const double f = (fhat - (double)fc->f_min[r]) / ((double)fc->f_max[r] - (double)fc->f_min[r]);
+  /* eta_i: the option's variant differs from the one in use (none in use: 0) */
+  const int32_t eta = fc->prev_variant[i] >= 0 && fc->variant[r] != fc->prev_variant[i];
+  const double margin = (double)fc->tau[i] + (double)fc->delta - f;
+  const double u = (double)fc->omega[i] * f * (double)fc->quality[r] -
+                   (double)fc->alpha * (double)eta * (double)fc->reload_cost[i] -
+                   (double)fc->beta * (margin > 0.0 ? margin * margin : 0.0);
+  if (fhat_out) *fhat_out = fhat;
+  if (f_out) *f_out = f;
+  /* the hard throughput floor f_i >= tau_i (inclusive) */
+  if (ok_out) *ok_out = f >= (double)fc->tau[i];
+  return u;
+}
+
+void orc_fc_local(const orc_problem *p, const orc_fc *fc, double *fhat, double *f, int32_t *ok,
+                  double *u) {
+  double zs[4];
+  fc_inputs(p, fc, zs);
+  for (int32_t i = 0; i < p->n_models; ++i)
+    for (int32_t o = 0; o < p->n_options[i]; ++o) {
+      const int64_t r = option_offset(p, i) + o;
+      u[r] = fc_term(p, fc, i, r, zs, &fhat[r], &f[r], &ok[r]);
+    }
+}
+
+double orc_fc_score_digits(const orc_problem *p, const orc_fc *fc, const int32_t *o, int32_t *feasible) {
+  double zs[4];
+  fc_inputs(p, fc, zs);
+  double J = 0.0, vram = 0.0;
+  int32_t floors = 1;
+  for (int32_t i = 0; i < p->n_models; ++i) {
+    const int64_t r = option_offset(p, i) + o[i];
+    int32_t ok;
+    J += fc_term(p, fc, i, r, zs, NULL, NULL, &ok);
+    floors = floors && ok;
+    vram += (double)p->demand[3 * r + 1];
+  }
+  int32_t feas = floors && vram <= (double)p->vram_cap;
+  if (isnan(J)) feas = 0;
+  if (feasible) *feasible = feas;
+  return feas ? J : -INFINITY;
+}
+
+void orc_fc_exhaustive(const orc_problem *p, const orc_fc *fc, uint64_t lo, uint64_t hi, int32_t k,
+                       uint64_t *topk_idx, double *topk_score, uint64_t *count, int32_t nthreads) {
+  for (int32_t j = 0; j < k; ++j) { topk_idx[j] = UINT64_MAX; topk_score[j] = -INFINITY; }
+  uint64_t total_count = 0;
+  const uint64_t size = orc_space_size(p);
+  if (hi > size) hi = size;
+  if (nthreads < 1) nthreads = 1;
+#ifdef _OPENMP
+#pragma omp parallel num_threads(nthreads)
+#endif
+  {
+    uint64_t *li = (uint64_t *)malloc(sizeof(uint64_t) * (size_t)k);
+    double *ls = (double *)malloc(sizeof(double) * (size_t)k);
+    for (int32_t j = 0; j < k; ++j) { li[j] = UINT64_MAX; ls[j] = -INFINITY; }
+    uint64_t c = 0;
+    int32_t o[64];
+#ifdef _OPENMP
+#pragma omp for schedule(dynamic, 4096)
+#endif
+    for (int64_t t = (int64_t)lo; t < (int64_t)hi; ++t) {
+      int32_t f = 0;
+      orc_decode(p, (uint64_t)t, o);
+      const double J = orc_fc_score_digits(p, fc, o, &f);
+      if (f) {
+        ++c;
+        topk_insert(k, li, ls, J, (uint64_t)t);
+      }
+    }
+#ifdef _OPENMP
+#pragma omp critical
+#endif
+    {
+      total_count += c;
+      for (int32_t j = 0; j < k; ++j)
+        if (li[j] != UINT64_MAX) topk_insert(k, topk_idx, topk_score, ls[j], li[j]);
+    }
+    free(li);
+    free(ls);
+  }
+  *count = total_count;
+}
+
+uint64_t orc_vram_feasible(const orc_problem *p, uint64_t lo, uint64_t hi, uint64_t *out, uint64_t cap) {
+  const uint64_t size = orc_space_size(p);
+  if (hi > size) hi = size;
+  uint64_t c = 0;
+  int32_t o[64];
+  for (uint64_t t = lo; t < hi; ++t) {
+    orc_decode(p, t, o);
+    double vram = 0.0;
+    for (int32_t i = 0; i < p->n_models; ++i) vram += (double)p->demand[3 * (option_offset(p, i) + o[i]) + 1];
+    /* Eq. 4: sum_i r_i^VRAM <= R; the others are removed when Lambda is built */
+    if (vram <= (double)p->vram_cap) {
+      if (c < cap) out[c] = t;
+      ++c;
+    }
+  }
+  return c;
+}

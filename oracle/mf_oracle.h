@@ -18,6 +18,11 @@
  *   orc_ga_init / orc_ga_step         pinned by operator properties (elitism,
  *                                     parent provenance, mutation rate, ranges)
  *   orc_ga_run                        parity unpinned beyond the operator level
+ *   orc_fc_local, orc_fc_score_digits,
+ *   orc_fc_exhaustive                 pinned (hand example, separable closed form,
+ *                                     reload term = alpha c, quadratic margin term,
+ *                                     linear case as one matrix product)
+ *   orc_vram_feasible                 pinned (two-pointer count, brute-force list)
  */
 #ifndef MF_ORACLE_H
 #define MF_ORACLE_H
@@ -93,6 +98,45 @@ void orc_ga_step(const orc_problem *p, const orc_ga_params *g, uint64_t seed, in
 /* Full GA: returns best fitness; best_genome[N]. */
 double orc_ga_run(const orc_problem *p, const orc_ga_params *g, uint64_t seed,
                   int32_t *best_genome, int32_t nthreads);
+
+/* ---------------------------------------------------------------------------
+ * Fixed-context mode (Sec. III-B: the observed state s_t = (rho_t, m_t, u_t) is
+ * held fixed during the search) with the utility of Eq. 3 and the constraints of
+ * Eq. 4: each predictor sees its own option and the observed aggregate state.
+ * ------------------------------------------------------------------------- */
+typedef struct {
+  const float *obs;            /* [4] observed aggregate state, raw units of the
+                                  aggregate (Sigma SM, Sigma VRAM, Sigma BW, N) */
+  const int32_t *variant;      /* [sum K_i] variant of each option */
+  const float *quality;        /* [sum K_i] Q of the option's variant */
+  const float *f_min;          /* [sum K_i] throughput extrema of the option's variant */
+  const float *f_max;
+  const float *omega;          /* [N] priority weights */
+  const float *tau;            /* [N] normalised throughput floors */
+  const float *reload_cost;    /* [N] c_i^rel */
+  const int32_t *prev_variant; /* [N] variant in use (-1: none) */
+  float alpha, beta, delta;
+} orc_fc;
+
+/* Per option row r (model-major, as local_feats): raw predicted throughput
+ * fhat[r], normalised f[r], floor flag ok[r] = (f >= tau_i) and the option's
+ * utility term u[r] = omega_i f Q - alpha eta c_i - beta max(0, tau_i + delta - f)^2. */
+void orc_fc_local(const orc_problem *p, const orc_fc *fc, double *fhat, double *f, int32_t *ok,
+                  double *u);
+
+/* J(lambda) of Eq. 3 in fixed-context mode (-inf, *feasible = 0, when a floor
+ * f_i >= tau_i or the VRAM bound of Eq. 4 fails). */
+double orc_fc_score_digits(const orc_problem *p, const orc_fc *fc, const int32_t *o, int32_t *feasible);
+
+/* Exhaustive fixed-context search over [lo, hi): top-k by (J desc, idx asc) and
+ * the feasible count; unfilled slots are (UINT64_MAX, -inf). */
+void orc_fc_exhaustive(const orc_problem *p, const orc_fc *fc, uint64_t lo, uint64_t hi, int32_t k,
+                       uint64_t *topk_idx, double *topk_score, uint64_t *count, int32_t nthreads);
+
+/* The VRAM-feasible joint configurations in [lo, hi) (Lambda with the
+ * VRAM-infeasible configurations removed), ascending; writes at most cap of
+ * them to out and returns how many there are. */
+uint64_t orc_vram_feasible(const orc_problem *p, uint64_t lo, uint64_t hi, uint64_t *out, uint64_t cap);
 
 #ifdef __cplusplus
 }

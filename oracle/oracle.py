@@ -50,6 +50,13 @@ class _Problem(C.Structure):
     ]
 
 
+class _FC(C.Structure):
+    _fields_ = [("obs", C.c_void_p), ("variant", C.c_void_p), ("quality", C.c_void_p),
+                ("f_min", C.c_void_p), ("f_max", C.c_void_p), ("omega", C.c_void_p),
+                ("tau", C.c_void_p), ("reload_cost", C.c_void_p), ("prev_variant", C.c_void_p),
+                ("alpha", C.c_float), ("beta", C.c_float), ("delta", C.c_float)]
+
+
 class _GAParams(C.Structure):
     _fields_ = [("pop", C.c_int32), ("gens", C.c_int32), ("tournament", C.c_int32),
                 ("mutation_p", C.c_double), ("elitism", C.c_int32)]
@@ -78,6 +85,12 @@ def _load():
             lib.orc_ga_init.argtypes = [P, G, u64, vp]; lib.orc_ga_init.restype = None
             lib.orc_ga_step.argtypes = [P, G, u64, i32, vp, vp, vp]; lib.orc_ga_step.restype = None
             lib.orc_ga_run.argtypes = [P, G, u64, vp, i32]; lib.orc_ga_run.restype = dbl
+            F = C.POINTER(_FC)
+            lib.orc_fc_local.argtypes = [P, F, vp, vp, vp, vp]; lib.orc_fc_local.restype = None
+            lib.orc_fc_score_digits.argtypes = [P, F, vp, vp]; lib.orc_fc_score_digits.restype = dbl
+            lib.orc_fc_exhaustive.argtypes = [P, F, u64, u64, i32, vp, vp, vp, i32]
+            lib.orc_fc_exhaustive.restype = None
+            lib.orc_vram_feasible.argtypes = [P, u64, u64, vp, u64]; lib.orc_vram_feasible.restype = u64
             _lib = lib
     return _lib
 
@@ -185,6 +198,59 @@ class Oracle:
         best = np.zeros(self.n, dtype=np.int32)
         J = self.lib.orc_ga_run(C.byref(self.p), C.byref(g), int(seed), _ptr(best), self.nthreads)
         return float(J), best
+
+
+    # -- fixed-context mode (Sec. III-B, Eq. 3, Eq. 4) ---------------------------
+    def _fc(self, fc: dict) -> _FC:
+        keep = {
+            "obs": np.ascontiguousarray(fc["obs"], dtype=np.float32),
+            "variant": np.ascontiguousarray(fc["variant"], dtype=np.int32),
+            "quality": np.ascontiguousarray(fc["quality"], dtype=np.float32),
+            "f_min": np.ascontiguousarray(fc["f_min"], dtype=np.float32),
+            "f_max": np.ascontiguousarray(fc["f_max"], dtype=np.float32),
+            "omega": np.ascontiguousarray(fc["omega"], dtype=np.float32),
+            "tau": np.ascontiguousarray(fc["tau"], dtype=np.float32),
+            "reload_cost": np.ascontiguousarray(fc["reload_cost"], dtype=np.float32),
+            "prev_variant": np.ascontiguousarray(fc["prev_variant"], dtype=np.int32),
+        }
+        self._fc_keep = keep
+        return _FC(*(_ptr(keep[k]) for k in ("obs", "variant", "quality", "f_min", "f_max", "omega", "tau",
+                                             "reload_cost", "prev_variant")),
+                   float(fc["alpha"]), float(fc["beta"]), float(fc["delta"]))
+
+    def fc_local(self, fc: dict):
+        """Per option row: (fhat, f, ok, u)."""
+        f_ = self._fc(fc)
+        rows = int(np.asarray(self._arr["n_options"]).sum())
+        fhat, f, u = (np.empty(rows) for _ in range(3))
+        ok = np.empty(rows, dtype=np.int32)
+        self.lib.orc_fc_local(C.byref(self.p), C.byref(f_), _ptr(fhat), _ptr(f), _ptr(ok), _ptr(u))
+        return fhat, f, ok.astype(bool), u
+
+    def fc_score_digits(self, fc: dict, digits):
+        f_ = self._fc(fc)
+        o = np.ascontiguousarray(digits, dtype=np.int32)
+        feas = np.zeros(1, dtype=np.int32)
+        J = self.lib.orc_fc_score_digits(C.byref(self.p), C.byref(f_), _ptr(o), _ptr(feas))
+        return float(J), bool(feas[0])
+
+    def fc_exhaustive(self, fc: dict, k: int, lo: int = 0, hi: int | None = None):
+        f_ = self._fc(fc)
+        hi = self.space_size() if hi is None else int(hi)
+        ti = np.empty(k, dtype=np.uint64)
+        ts = np.empty(k, dtype=np.float64)
+        cnt = np.zeros(1, dtype=np.uint64)
+        self.lib.orc_fc_exhaustive(C.byref(self.p), C.byref(f_), int(lo), hi, int(k), _ptr(ti), _ptr(ts),
+                                   _ptr(cnt), self.nthreads)
+        return ti, ts, int(cnt[0])
+
+    def vram_feasible(self, lo: int = 0, hi: int | None = None, cap: int | None = None):
+        """(count, ascending list of the first min(count, cap) VRAM-feasible indices)."""
+        hi = self.space_size() if hi is None else int(hi)
+        cap = (hi - int(lo)) if cap is None else int(cap)
+        out = np.empty(max(cap, 1), dtype=np.uint64)
+        c = int(self.lib.orc_vram_feasible(C.byref(self.p), int(lo), hi, _ptr(out), cap))
+        return c, out[:min(c, cap)]
 
 
 def splitmix64(seed: int, ctr: int) -> int:

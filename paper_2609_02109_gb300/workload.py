@@ -224,6 +224,47 @@ def integer_landscape(n_options, seed: int, vram_cap: float, objective="weighted
     )
 
 
+# stream purposes of the fixed-context inputs
+P_OBS, P_FMIN, P_FMAX, P_TAU, P_PREV = range(13, 18)
+
+
+def fc_scenario(prob: dict, seed: int) -> dict:
+    """Inputs of the fixed-context mode (observed state, per-option variant data, the
+    utility constants of Eq. 3) for a problem drawn by make_problem.
+
+    Model i alternates between an LLM-like model (two variants, FP16 / AWQ, quality
+    1.000 / 0.979, reload cost 30 s) and a vision-like one (three variants, n / s / m,
+    quality 0.73 / 0.96 / 1.00, reload cost 5 s) -- the paper's values (Sec. II).
+    Option o of model i belongs to variant o mod V_i.  The per-variant throughput
+    extrema stand in for the profiling extrema: f_min ~ U(-1, -0.2), f_max ~
+    U(0.2, 1) (the synthetic predictors' outputs are of order 0.3).  The observed
+    state is the aggregate of a typical configuration: SM share U(0.2, 0.4) N, VRAM
+    U(5, 15) N GB, BW U(500, 1000) N GB/s.  Floors tau_i ~ U(-0.1, 0.15); the variant
+    in use is uniform, or none (-1) with probability 1/4.  omega_i = 1, alpha = 1/60,
+    beta = 5, delta = 0.05 (Sec. II)."""
+    k = np.asarray(prob["n_options"], dtype=np.int64)
+    n = int(k.size)
+    llm = np.arange(n) % 2 == 0
+    nv = np.where(llm, 2, 3)
+    variant = np.concatenate([np.arange(int(k[i])) % nv[i] for i in range(n)]).astype(np.int32)
+    qual = [np.array([1.000, 0.979]) if llm[i] else np.array([0.73, 0.96, 1.00]) for i in range(n)]
+    quality = np.concatenate([qual[i][np.arange(int(k[i])) % nv[i]] for i in range(n)]).astype(np.float32)
+    fmin_v = [uniform(seed, P_FMIN, i, int(nv[i]), -1.0, -0.2) for i in range(n)]
+    fmax_v = [uniform(seed, P_FMAX, i, int(nv[i]), 0.2, 1.0) for i in range(n)]
+    f_min = np.concatenate([fmin_v[i][np.arange(int(k[i])) % nv[i]] for i in range(n)]).astype(np.float32)
+    f_max = np.concatenate([fmax_v[i][np.arange(int(k[i])) % nv[i]] for i in range(n)]).astype(np.float32)
+    o = uniform(seed, P_OBS, 0, 3, 0.0, 1.0).astype(np.float64)
+    obs = np.array([(0.2 + 0.2 * o[0]) * n, (5.0 + 10.0 * o[1]) * n, (500.0 + 500.0 * o[2]) * n, n],
+                   dtype=np.float32)
+    pz = stream_u64(stream_key(seed, P_PREV, 0), 2 * n)
+    prev = np.array([-1 if (pz[2 * i] >> np.uint64(62)) == 0 else int((pz[2 * i + 1] >> np.uint64(32)) % np.uint64(nv[i]))
+                     for i in range(n)], dtype=np.int32)
+    return dict(obs=obs, variant=variant, quality=quality, f_min=f_min, f_max=f_max,
+                omega=np.ones(n, dtype=np.float32), tau=uniform(seed, P_TAU, 0, n, -0.1, 0.15),
+                reload_cost=np.where(llm, 30.0, 5.0).astype(np.float32), prev_variant=prev,
+                alpha=1.0 / 60.0, beta=5.0, delta=0.05)
+
+
 GA_SCENARIO_SEEDS = tuple(range(100, 108))
 GA_RUN_SEEDS = tuple(range(1000, 1050))
 
