@@ -208,6 +208,58 @@ mf_status mf_ga_step(mf_ctx *ctx, const mf_ga_params *g, uint64_t seed, int32_t 
 mf_status mf_ga_run(mf_ctx *ctx, const mf_ga_params *g, uint64_t seed, int32_t *best_genome,
                     float *best_fitness, void *stream);
 
+/* ---------------------------------------------------------------------------
+ * Fixed-context mode (Sec. III-B): the observed GPU state s_t is held fixed during
+ * the search, so predictor i sees its own option and the observed state only, and
+ * the utility of Eq. 3 separates into one term per model:
+ *   J = sum_i [omega_i f_i Q_i - alpha eta_i c_i - beta max(0, tau_i + delta - f_i)^2]
+ * with f_i = (fhat_i - f_min) / (f_max - f_min) the per-variant min-max normalised
+ * predicted throughput (fhat_i: the predictor's throughput output) and eta_i = 1 when
+ * option i's variant differs from the variant in use.  Constraints (Eq. 4): the
+ * summed VRAM of the chosen options <= vram_cap and f_i >= tau_i for every model;
+ * otherwise J = -inf.
+ * ------------------------------------------------------------------------- */
+typedef struct {
+  const float *obs;            /* [4] observed state in the aggregate's raw units
+                                  (Sigma SM share, Sigma VRAM GB, Sigma BW GB/s, N);
+                                  fed to the predictors scaled by agg_scale */
+  const int32_t *variant;      /* [sum K_i] variant of each option (>= 0), model-major */
+  const float *quality;        /* [sum K_i] Q of the option's variant */
+  const float *f_min;          /* [sum K_i] throughput extrema of the option's variant, */
+  const float *f_max;          /*           f_max > f_min */
+  const float *omega;          /* [N] priority weights */
+  const float *tau;            /* [N] floors on the normalised throughput */
+  const float *reload_cost;    /* [N] c_i^rel */
+  const int32_t *prev_variant; /* [N] variant in use, -1 for none (eta_i = 0) */
+  float alpha, beta, delta;    /* paper: 1/60, 5.0, 0.05 */
+} mf_fc_params;
+
+/* Evaluate the sum K_i local predictions under p->obs with the fp32 predictor and
+ * build the per-option table (fhat, f, floor flag, utility term) on the device; the
+ * context keeps it for mf_fc_search until the next call.  Host arrays, copied.
+ * Synchronous on `stream`.  MF_EINVAL: NULL arrays, f_max <= f_min, variant < 0,
+ * prev_variant < -1, non-finite constants. */
+mf_status mf_fc_set(mf_ctx *ctx, const mf_fc_params *p, void *stream);
+
+/* Copy the table of the last mf_fc_set into caller-owned device arrays of sum K_i
+ * entries (model-major; any may be NULL): fhat, f, u (the option's term of J), ok
+ * (1: f >= tau_i).  Asynchronous on `stream`.  MF_EINVAL before mf_fc_set. */
+mf_status mf_fc_table(mf_ctx *ctx, float *d_fhat, float *d_f, float *d_u, uint8_t *d_ok, void *stream);
+
+/* Fixed-context exhaustive search over [lo, hi): J(lambda) = sum of the options'
+ * terms (fp32, model order), the same result contract as mf_search_range (top-k by
+ * J desc then index asc, feasible count, empty slots (UINT64_MAX, -inf)).  An
+ * ALU-bound table-lookup scan.  MF_EINVAL before mf_fc_set. */
+mf_status mf_fc_search(mf_ctx *ctx, uint64_t lo, uint64_t hi, int32_t k, uint64_t chunk, mf_result *out,
+                       void *stream);
+
+/* Lambda without its VRAM-infeasible configurations (Eq. 4 applied when Lambda is
+ * built): writes the ascending indices of [lo, hi) whose summed VRAM <= vram_cap to
+ * d_out (device, capacity cap; indices beyond cap are counted, not written) and
+ * their number to *count (host).  Synchronous. */
+mf_status mf_vram_feasible(mf_ctx *ctx, uint64_t lo, uint64_t hi, uint64_t *d_out, uint64_t cap,
+                           uint64_t *count, void *stream);
+
 /* Read the context's instrumentation (see mf_stats). */
 mf_status mf_get_stats(const mf_ctx *ctx, mf_stats *out);
 

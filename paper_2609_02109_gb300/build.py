@@ -18,7 +18,7 @@ BUILD_DIR = os.path.join(HERE, "_build")
 LIB_PATH = os.path.join(OUT_DIR, "libmfsched.so")
 ROOT = os.path.dirname(HERE)
 
-SOURCES = ["mf_api.cu", "k_f32.cu", "k_select.cu", "k_ga.cu", "k_tc.cu", "mf_noalloc.cu"]
+SOURCES = ["mf_api.cu", "k_f32.cu", "k_select.cu", "k_ga.cu", "k_tc.cu", "k_fc.cu", "mf_noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

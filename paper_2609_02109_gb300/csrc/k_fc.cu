@@ -1,0 +1,481 @@
+// Fixed-context mode (arXiv 2609.02109, Sec. III-B): the observed GPU state s_t is
+// held fixed during the search, so predictor g_i(lambda_i, s_t) depends on model i's
+// option only.  The sum K_i local predictions are evaluated once (k_fc_local) into a
+// per-option table of the utility term of Eq. 3,
+//   u = omega_i f Q - alpha eta c_i - beta max(0, tau_i + delta - f)^2,
+//   f = (fhat - f_min) / (f_max - f_min)   (per-variant normalisation),
+// and a joint configuration's J is the sum of its options' terms (Eq. 3), -inf when a
+// floor f_i >= tau_i or the VRAM bound of Eq. 4 fails.  The exhaustive search is then
+// a table-lookup scan (k_fc_scan, ALU-bound); k_vram_count / k_vram_write build the
+// VRAM-feasible space (Lambda without its VRAM-infeasible configurations) as an
+// ascending index list.
+#include <cmath>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "mf_internal.cuh"
+
+namespace mf {
+
+// Device layout of mf_ctx::d_fc.
+struct FcLayout {
+  float2* tab;       // [sumK] (u, or -inf below the floor; VRAM of the option)
+  float* fhat;       // [sumK]
+  float* f;          // [sumK]
+  float* u;          // [sumK]
+  uint8_t* ok;       // [sumK]
+  // inputs, copied
+  float* obs;        // [4]
+  int32_t* variant;  // [sumK]
+  float* quality;    // [sumK]
+  float* f_min;      // [sumK]
+  float* f_max;      // [sumK]
+  float* omega;      // [N]
+  float* tau;        // [N]
+  float* cost;       // [N]
+  int32_t* prev;     // [N]
+};
+
+static size_t fc_bytes(int sumK, int N, FcLayout* L, char* base) {
+  size_t o = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = o;
+    o = (o + bytes + 255) / 256 * 256;
+    return base ? base + at : nullptr;
+  };
+  char* p;
+  p = take(sizeof(float2) * sumK); if (L) L->tab = (float2*)p;
+  p = take(sizeof(float) * sumK); if (L) L->fhat = (float*)p;
+  p = take(sizeof(float) * sumK); if (L) L->f = (float*)p;
+  p = take(sizeof(float) * sumK); if (L) L->u = (float*)p;
+  p = take(sumK); if (L) L->ok = (uint8_t*)p;
+  p = take(sizeof(float) * 4); if (L) L->obs = (float*)p;
+  p = take(sizeof(int32_t) * sumK); if (L) L->variant = (int32_t*)p;
+  p = take(sizeof(float) * sumK); if (L) L->quality = (float*)p;
+  p = take(sizeof(float) * sumK); if (L) L->f_min = (float*)p;
+  p = take(sizeof(float) * sumK); if (L) L->f_max = (float*)p;
+  p = take(sizeof(float) * N); if (L) L->omega = (float*)p;
+  p = take(sizeof(float) * N); if (L) L->tau = (float*)p;
+  p = take(sizeof(float) * N); if (L) L->cost = (float*)p;
+  p = take(sizeof(int32_t) * N); if (L) L->prev = (int32_t*)p;
+  return o;
+}
+
+struct FcConst {
+  float alpha, beta, delta;
+};
+
+// ---------------------------------------------------------------------------
+// Local predictions: one CTA per option row.  z = [x_i(o) | obs * s_A]; the hidden
+// layers spread their units over the threads; the throughput head reduces over
+// warp 0.  Thread 0 forms f, the floor flag and u.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256)
+k_fc_local(const Params P, const FcLayout L, const FcConst C) {
+  __shared__ float z[MF_MAX_D_LOCAL + 4];
+  __shared__ float h1[MF_MAX_HIDDEN], h2[MF_MAX_HIDDEN];
+  __shared__ int s_model;
+  const int r = blockIdx.x, tid = threadIdx.x;
+  const int N = P.n_models;
+  if (tid == 0) {
+    int m = 0;
+    for (int i = 0; i < N; ++i)
+      if (r >= pick(P.off, i)) m = i;
+    s_model = m;
+  }
+  const int dl = P.d_local, din = P.d_in, H1 = P.h1, H2 = P.h2;
+  for (int k = tid; k < dl; k += blockDim.x) z[k] = P.x[(size_t)r * dl + k];
+  if (tid < 4) z[dl + tid] = L.obs[tid] * P.agg_scale[tid];
+  __syncthreads();
+  const int m = s_model;
+  const float* w = P.w32 + (size_t)m * P.per_model;
+  const float* W1 = w;
+  const float* b1 = W1 + (size_t)H1 * din;
+  for (int j = tid; j < H1; j += blockDim.x) {
+    float s = b1[j];
+    for (int k = 0; k < din; ++k) s = fmaf(W1[(size_t)j * din + k], z[k], s);
+    h1[j] = relu(s);
+  }
+  __syncthreads();
+  const float* next = b1 + H1;
+  const float* h = h1;
+  int hl = H1;
+  if (H2 > 0) {
+    const float* W2 = next;
+    const float* b2 = W2 + (size_t)H2 * H1;
+    for (int j = tid; j < H2; j += blockDim.x) {
+      float s = b2[j];
+      for (int k = 0; k < H1; ++k) s = fmaf(W2[(size_t)j * H1 + k], h1[k], s);
+      h2[j] = relu(s);
+    }
+    __syncthreads();
+    next = b2 + H2;
+    h = h2;
+    hl = H2;
+  }
+  if (tid < 32) {
+    const float* W3 = next;  // row 0: the throughput head
+    float s = 0.f;
+    for (int k = tid; k < hl; k += 32) s = fmaf(W3[k], h[k], s);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    if (tid == 0) {
+      const float fhat = out_act(P, s + W3[2 * hl]);
+      const float f = (fhat - L.f_min[r]) / (L.f_max[r] - L.f_min[r]);
+      const float tau = L.tau[m];
+      const bool ok = f >= tau;
+      const float eta = (L.prev[m] >= 0 && L.variant[r] != L.prev[m]) ? 1.f : 0.f;
+      const float margin = tau + C.delta - f;
+      const float u = L.omega[m] * f * L.quality[r] - C.alpha * eta * L.cost[m] -
+                      C.beta * (margin > 0.f ? margin * margin : 0.f);
+      L.fhat[r] = fhat;
+      L.f[r] = f;
+      L.u[r] = u;
+      L.ok[r] = ok ? 1 : 0;
+      L.tab[r] = make_float2(ok ? u : -INFINITY, P.dem[r].y);
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Table-lookup scan: one candidate per thread and step; digits advance by the grid
+// stride with carries.  Per-CTA running top-k as in the fp32 scorer.
+// ---------------------------------------------------------------------------
+constexpr int kFcThreads = 512;
+
+struct FcScan {
+  const float2* tab;
+  uint32_t step[MF_MAX_MODELS];  // mixed-radix digits of the grid stride (grid x threads)
+};
+
+__global__ void __launch_bounds__(kFcThreads, 1)
+k_fc_scan(const Params P, const FcScan S, const RangeArgs R) {
+  extern __shared__ __align__(16) unsigned char sm[];
+  const int N = P.n_models;
+  const int sumK = pick(P.off, N - 1) + pick(P.K, N - 1);
+  float2* tab = reinterpret_cast<float2*>(sm);
+  unsigned char* q = sm + (((size_t)sumK * sizeof(float2) + 15) & ~(size_t)15);
+  const int tid = threadIdx.x;
+  CtaTopK tk;
+  tk.li = reinterpret_cast<uint64_t*>(q); q += sizeof(uint64_t) * R.k;
+  tk.ni = reinterpret_cast<uint64_t*>(q); q += sizeof(uint64_t) * R.k;
+  tk.qi = reinterpret_cast<uint64_t*>(q); q += sizeof(uint64_t) * kFcThreads;
+  tk.ls = reinterpret_cast<float*>(q); q += sizeof(float) * R.k;
+  tk.ns = reinterpret_cast<float*>(q); q += sizeof(float) * R.k;
+  tk.qs = reinterpret_cast<float*>(q); q += sizeof(float) * kFcThreads;
+  tk.qn = reinterpret_cast<int*>(q);
+  tk.k = R.k;
+  for (int e = tid; e < sumK; e += blockDim.x) tab[e] = S.tab[e];
+  const size_t gl = (size_t)blockIdx.x * R.k;
+  for (int e = tid; e < R.k; e += blockDim.x) {
+    tk.ls[e] = R.first ? -INFINITY : R.lists_s[gl + e];
+    tk.li[e] = R.first ? kEmptyIdx : R.lists_i[gl + e];
+  }
+  if (tid == 0) *tk.qn = 0;
+  // this thread's first candidate and its option rows
+  const uint64_t t0 = (uint64_t)blockIdx.x * blockDim.x + tid;
+  int row[MF_MAX_MODELS];
+  {
+    const uint64_t idx0 = R.base + (t0 < R.len ? t0 : 0);
+#pragma unroll
+    for (int i = 0; i < MF_MAX_MODELS; ++i)
+      if (i < N) row[i] = pick(P.off, i) + (int)((idx0 / pick(P.stride, i)) % (uint64_t)pick(P.K, i));
+  }
+  __syncthreads();
+  float thr_s = tk.ls[R.k - 1];
+  uint64_t thr_i = tk.li[R.k - 1];
+  const float cap = P.vram_cap;
+  unsigned int my_count = 0;
+  const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
+  for (uint64_t base = (uint64_t)blockIdx.x * blockDim.x; base < R.len; base += stride) {
+    const uint64_t t = base + tid;
+    const bool valid = t < R.len;
+    float J = 0.f, V = 0.f;
+#pragma unroll
+    for (int i = 0; i < MF_MAX_MODELS; ++i)
+      if (i < N) {
+        const float2 e = tab[row[i]];
+        J += e.x;
+        V += e.y;
+      }
+    // -inf below a floor; NaN compares false
+    const bool feas = valid && V <= cap && J > -INFINITY;
+    const uint64_t idx = R.base + t;
+    my_count += feas ? 1u : 0u;
+    const bool push = feas && precedes(J, idx, thr_s, thr_i);
+    if (push) {
+      const int pos = atomicAdd(tk.qn, 1);
+      tk.qs[pos] = J;
+      tk.qi[pos] = idx;
+    }
+    if (__syncthreads_or(push)) {  // block-uniform
+      topk_merge(tk, tid, blockDim.x, [] __device__() { __syncthreads(); });
+      thr_s = tk.ls[R.k - 1];
+      thr_i = tk.li[R.k - 1];
+    }
+    // advance the digits by the stride, last model first
+    uint32_t carry = 0;
+#pragma unroll
+    for (int i = MF_MAX_MODELS - 1; i >= 0; --i)
+      if (i < N) {
+        const int off = pick(P.off, i);
+        const uint32_t K = (uint32_t)pick(P.K, i);
+        uint32_t d = (uint32_t)(row[i] - off) + S.step[i] + carry;
+        carry = d >= K;
+        if (carry) d -= K;
+        row[i] = off + (int)d;
+      }
+  }
+  for (int e = tid; e < R.k; e += blockDim.x) {
+    R.lists_s[gl + e] = tk.ls[e];
+    R.lists_i[gl + e] = tk.li[e];
+  }
+  unsigned int c = my_count;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
+  if ((tid & 31) == 0 && c) atomicAdd(R.count, (unsigned long long)c);
+}
+
+// ---------------------------------------------------------------------------
+// VRAM-feasible space: CTA b scans the contiguous segment [b*seg, (b+1)*seg) of the
+// range, in steps of 512 consecutive candidates.  k_vram_count counts; after an
+// exclusive scan of the counts, k_vram_write writes each CTA's indices in order.
+// ---------------------------------------------------------------------------
+constexpr int kVramThreads = 512;
+
+struct VramArgs {
+  uint64_t lo, len, seg;
+  uint32_t step[MF_MAX_MODELS];   // mixed-radix digits of 512
+  unsigned long long* counts;     // [grid]
+  uint64_t* out;
+  uint64_t cap;
+};
+
+template <bool WRITE>
+__global__ void __launch_bounds__(kVramThreads)
+k_vram(const Params P, const VramArgs A) {
+  extern __shared__ __align__(16) float vr[];  // [sumK] VRAM of each option
+  __shared__ unsigned int s_warp[kVramThreads / 32];
+  __shared__ unsigned long long s_base;
+  const int N = P.n_models;
+  const int sumK = pick(P.off, N - 1) + pick(P.K, N - 1);
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  for (int e = tid; e < sumK; e += blockDim.x) vr[e] = P.dem[e].y;
+  const uint64_t s0 = (uint64_t)blockIdx.x * A.seg;
+  const uint64_t s1 = s0 + A.seg < A.len ? s0 + A.seg : A.len;
+  int row[MF_MAX_MODELS];
+  {
+    const uint64_t idx0 = A.lo + (s0 + tid < A.len ? s0 + tid : 0);
+#pragma unroll
+    for (int i = 0; i < MF_MAX_MODELS; ++i)
+      if (i < N) row[i] = pick(P.off, i) + (int)((idx0 / pick(P.stride, i)) % (uint64_t)pick(P.K, i));
+  }
+  if (tid == 0) s_base = WRITE ? A.counts[blockIdx.x] : 0ull;
+  __syncthreads();
+  unsigned long long mine = 0;
+  for (uint64_t b = s0; b < s1; b += kVramThreads) {
+    const uint64_t t = b + tid;
+    float V = 0.f;
+#pragma unroll
+    for (int i = 0; i < MF_MAX_MODELS; ++i)
+      if (i < N) V += vr[row[i]];
+    const bool ok = t < s1 && V <= P.vram_cap;
+    if (WRITE) {
+      // ascending positions: this warp's earlier lanes, then the earlier warps
+      const unsigned int bal = __ballot_sync(0xffffffffu, ok);
+      if (lane == 0) s_warp[warp] = __popc(bal);
+      __syncthreads();
+      unsigned int before = __popc(bal & ((1u << lane) - 1u));
+      unsigned int total = 0;
+      for (int w = 0; w < kVramThreads / 32; ++w) {
+        if (w < warp) before += s_warp[w];
+        total += s_warp[w];
+      }
+      const unsigned long long pos = s_base + before;
+      if (ok && pos < A.cap) A.out[pos] = A.lo + t;
+      __syncthreads();
+      if (tid == 0) s_base += total;
+    } else {
+      mine += ok ? 1ull : 0ull;
+    }
+    uint32_t carry = 0;
+#pragma unroll
+    for (int i = MF_MAX_MODELS - 1; i >= 0; --i)
+      if (i < N) {
+        const int off = pick(P.off, i);
+        const uint32_t K = (uint32_t)pick(P.K, i);
+        uint32_t d = (uint32_t)(row[i] - off) + A.step[i] + carry;
+        carry = d >= K;
+        if (carry) d -= K;
+        row[i] = off + (int)d;
+      }
+  }
+  if (!WRITE) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) mine += __shfl_xor_sync(0xffffffffu, mine, o);
+    if (lane == 0) atomicAdd(&A.counts[blockIdx.x], mine);
+  }
+}
+
+// Exclusive scan of n counts in place (one CTA; n <= 4096); total to *total.
+__global__ void __launch_bounds__(1024)
+k_scan_counts(unsigned long long* c, int n, unsigned long long* total) {
+  __shared__ unsigned long long s[4096];
+  for (int e = threadIdx.x; e < n; e += blockDim.x) s[e] = c[e];
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    unsigned long long run = 0;
+    for (int e = 0; e < n; ++e) {
+      const unsigned long long v = s[e];
+      s[e] = run;
+      run += v;
+    }
+    *total = run;
+  }
+  __syncthreads();
+  for (int e = threadIdx.x; e < n; e += blockDim.x) c[e] = s[e];
+}
+
+static void radix_digits(const Params& P, uint64_t v, uint32_t* step) {
+  v %= P.total;
+  for (int i = P.n_models - 1; i >= 0; --i) {
+    step[i] = (uint32_t)(v % (uint64_t)P.K[i]);
+    v /= (uint64_t)P.K[i];
+  }
+}
+
+int fc_grid(const mf_ctx* c) { return c->num_sms; }
+
+mf_status fc_search_chunk(mf_ctx* c, const RangeArgs& a, cudaStream_t s) {
+  FcLayout L;
+  fc_bytes(c->sumK, c->P.n_models, &L, (char*)c->d_fc);
+  FcScan S{};
+  S.tab = L.tab;
+  radix_digits(c->P, (uint64_t)fc_grid(c) * kFcThreads, S.step);
+  const size_t smem = (((size_t)c->sumK * sizeof(float2) + 15) & ~(size_t)15) +
+                      (sizeof(uint64_t) + sizeof(float)) * (2 * (size_t)a.k + kFcThreads) + 16;
+  if (smem > 227 * 1024) {
+    set_error("fixed-context search: top-k lists do not fit shared memory; use a smaller k");
+    return MF_EUNSUPPORTED;
+  }
+  MF_CUDA(cudaFuncSetAttribute(k_fc_scan, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+  k_fc_scan<<<fc_grid(c), kFcThreads, smem, s>>>(c->P, S, a);
+  MF_CUDA(cudaGetLastError());
+  return MF_OK;
+}
+
+}  // namespace mf
+
+using namespace mf;
+
+static mf_status fc_einval(const std::string& m) {
+  set_error(m);
+  return MF_EINVAL;
+}
+
+mf_status mf_fc_set(mf_ctx* ctx, const mf_fc_params* p, void* stream) {
+  set_error("");
+  if (!ctx || !p) return fc_einval("NULL argument");
+  if (!p->obs || !p->variant || !p->quality || !p->f_min || !p->f_max || !p->omega || !p->tau ||
+      !p->reload_cost || !p->prev_variant)
+    return fc_einval("mf_fc_params: every array is required");
+  const int N = ctx->P.n_models, sumK = ctx->sumK;
+  for (int r = 0; r < sumK; ++r) {
+    if (!(p->f_max[r] > p->f_min[r])) return fc_einval("mf_fc_params: f_max must exceed f_min for every option");
+    if (p->variant[r] < 0) return fc_einval("mf_fc_params: variants must be >= 0");
+  }
+  for (int i = 0; i < N; ++i)
+    if (p->prev_variant[i] < -1) return fc_einval("mf_fc_params: prev_variant must be >= -1");
+  if (!std::isfinite(p->alpha) || !std::isfinite(p->beta) || !std::isfinite(p->delta))
+    return fc_einval("mf_fc_params: alpha, beta and delta must be finite");
+  DeviceGuard guard(ctx->device);
+  cudaStream_t s = (cudaStream_t)stream;
+  const size_t bytes = fc_bytes(sumK, N, nullptr, nullptr);
+  if (!ctx->d_fc) MF_CUDA(cudaMalloc(&ctx->d_fc, bytes));
+  FcLayout L;
+  fc_bytes(sumK, N, &L, (char*)ctx->d_fc);
+  // inputs to the device (pinned staging, one copy each, then a synchronisation)
+  std::vector<unsigned char> host(bytes);
+  auto put = [&](void* dev, const void* src, size_t n) {
+    std::memcpy(host.data() + ((char*)dev - (char*)ctx->d_fc), src, n);
+  };
+  put(L.obs, p->obs, sizeof(float) * 4);
+  put(L.variant, p->variant, sizeof(int32_t) * sumK);
+  put(L.quality, p->quality, sizeof(float) * sumK);
+  put(L.f_min, p->f_min, sizeof(float) * sumK);
+  put(L.f_max, p->f_max, sizeof(float) * sumK);
+  put(L.omega, p->omega, sizeof(float) * N);
+  put(L.tau, p->tau, sizeof(float) * N);
+  put(L.cost, p->reload_cost, sizeof(float) * N);
+  put(L.prev, p->prev_variant, sizeof(int32_t) * N);
+  const size_t in_lo = (char*)L.obs - (char*)ctx->d_fc;
+  MF_CUDA(cudaMemcpyAsync((char*)ctx->d_fc + in_lo, host.data() + in_lo, bytes - in_lo, cudaMemcpyHostToDevice, s));
+  const FcConst C{p->alpha, p->beta, p->delta};
+  k_fc_local<<<sumK, 256, 0, s>>>(ctx->P, L, C);
+  MF_CUDA(cudaGetLastError());
+  MF_CUDA(cudaStreamSynchronize(s));
+  ctx->fc_ready = 1;
+  return MF_OK;
+}
+
+mf_status mf_fc_table(mf_ctx* ctx, float* d_fhat, float* d_f, float* d_u, uint8_t* d_ok, void* stream) {
+  set_error("");
+  if (!ctx) return fc_einval("NULL argument");
+  if (!ctx->fc_ready) return fc_einval("mf_fc_set has not been called on this context");
+  DeviceGuard guard(ctx->device);
+  cudaStream_t s = (cudaStream_t)stream;
+  FcLayout L;
+  fc_bytes(ctx->sumK, ctx->P.n_models, &L, (char*)ctx->d_fc);
+  const size_t n = (size_t)ctx->sumK;
+  if (d_fhat) MF_CUDA(cudaMemcpyAsync(d_fhat, L.fhat, sizeof(float) * n, cudaMemcpyDeviceToDevice, s));
+  if (d_f) MF_CUDA(cudaMemcpyAsync(d_f, L.f, sizeof(float) * n, cudaMemcpyDeviceToDevice, s));
+  if (d_u) MF_CUDA(cudaMemcpyAsync(d_u, L.u, sizeof(float) * n, cudaMemcpyDeviceToDevice, s));
+  if (d_ok) MF_CUDA(cudaMemcpyAsync(d_ok, L.ok, n, cudaMemcpyDeviceToDevice, s));
+  return MF_OK;
+}
+
+mf_status mf_vram_feasible(mf_ctx* ctx, uint64_t lo, uint64_t hi, uint64_t* d_out, uint64_t cap,
+                           uint64_t* count, void* stream) {
+  set_error("");
+  if (!ctx || !count) return fc_einval("NULL argument");
+  if (lo > hi || hi > ctx->P.total) return fc_einval("need lo <= hi <= |Lambda|");
+  if (cap > 0 && !d_out) return fc_einval("d_out is NULL");
+  DeviceGuard guard(ctx->device);
+  cudaStream_t s = (cudaStream_t)stream;
+  const uint64_t len = hi - lo;
+  // segments of whole steps, at most 4096 CTAs
+  const uint64_t steps = (len + kVramThreads - 1) / kVramThreads;
+  uint64_t grid = 4ull * ctx->num_sms;
+  if (grid > steps) grid = steps > 0 ? steps : 1;
+  const uint64_t seg = ((steps + grid - 1) / grid) * kVramThreads;
+  grid = len > 0 ? (len + seg - 1) / seg : 1;
+  mf_status st = ensure_scratch(ctx, sizeof(unsigned long long) * (grid + 1));
+  if (st != MF_OK) return st;
+  unsigned long long* counts = (unsigned long long*)ctx->d_scratch;
+  VramArgs A{};
+  A.lo = lo;
+  A.len = len;
+  A.seg = seg;
+  radix_digits(ctx->P, kVramThreads, A.step);
+  A.counts = counts;
+  A.out = d_out;
+  A.cap = cap;
+  const size_t smem = sizeof(float) * (size_t)ctx->sumK;
+  MF_CUDA(cudaMemsetAsync(counts, 0, sizeof(unsigned long long) * (grid + 1), s));
+  k_vram<false><<<(unsigned)grid, kVramThreads, smem, s>>>(ctx->P, A);
+  MF_CUDA(cudaGetLastError());
+  k_scan_counts<<<1, 1024, 0, s>>>(counts, (int)grid, counts + grid);
+  MF_CUDA(cudaGetLastError());
+  if (cap > 0) {
+    k_vram<true><<<(unsigned)grid, kVramThreads, smem, s>>>(ctx->P, A);
+    MF_CUDA(cudaGetLastError());
+  }
+  st = ensure_host_stage(ctx, sizeof(unsigned long long));
+  if (st != MF_OK) return st;
+  unsigned long long* h = (unsigned long long*)ctx->h_stage;
+  MF_CUDA(cudaMemcpyAsync(h, counts + grid, sizeof(unsigned long long), cudaMemcpyDeviceToHost, s));
+  MF_CUDA(cudaStreamSynchronize(s));
+  *count = *h;
+  return MF_OK;
+}

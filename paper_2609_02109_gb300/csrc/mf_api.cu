@@ -22,18 +22,6 @@ static mf_status einval(const std::string& msg) {
   return MF_EINVAL;
 }
 
-// Makes the context's device current for the scope of an API call.
-struct DeviceGuard {
-  int prev = -1;
-  bool changed = false;
-  explicit DeviceGuard(int dev) {
-    if (cudaGetDevice(&prev) == cudaSuccess && prev != dev) changed = cudaSetDevice(dev) == cudaSuccess;
-  }
-  ~DeviceGuard() {
-    if (changed) cudaSetDevice(prev);
-  }
-};
-
 static size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
 mf_status ensure_scratch(mf_ctx* c, size_t bytes) {
@@ -71,6 +59,7 @@ static void free_ctx(mf_ctx* c) {
   cudaFree(c->d_status);
   cudaFree(c->d_tc);
   cudaFree(c->d_partial);
+  cudaFree(c->d_fc);
   cudaFree(c->d_scratch);
   cudaFree(c->d_pop[0]);
   cudaFree(c->d_pop[1]);
@@ -314,9 +303,27 @@ static mf_status read_status(mf_ctx* ctx, cudaStream_t s, uint32_t* word, bool c
   return MF_OK;
 }
 
+// The exhaustive-search driver: per-CTA running lists over chunks of [lo, hi), their
+// merge, the fp32 re-scoring of a bf16 shortlist, the result.  fc: the fixed-context
+// table-lookup scan instead of the predictors.
+static mf_status search_impl(mf_ctx* ctx, uint64_t lo, uint64_t hi, int32_t k, uint64_t chunk,
+                             mf_result* out, void* stream, bool fc);
+
 mf_status mf_search_range(mf_ctx* ctx, uint64_t lo, uint64_t hi, int32_t k, uint64_t chunk,
                           mf_result* out, void* stream) {
   g_last_error.clear();
+  return search_impl(ctx, lo, hi, k, chunk, out, stream, false);
+}
+
+mf_status mf_fc_search(mf_ctx* ctx, uint64_t lo, uint64_t hi, int32_t k, uint64_t chunk, mf_result* out,
+                       void* stream) {
+  g_last_error.clear();
+  if (ctx && !ctx->fc_ready) return einval("mf_fc_set has not been called on this context");
+  return search_impl(ctx, lo, hi, k, chunk, out, stream, true);
+}
+
+static mf_status search_impl(mf_ctx* ctx, uint64_t lo, uint64_t hi, int32_t k, uint64_t chunk,
+                             mf_result* out, void* stream, bool fc) {
   if (!ctx || !out) return einval("NULL argument");
   if (k < 1 || k > MF_MAX_TOPK) return einval("k must be in 1..1024");
   if (lo > hi || hi > ctx->P.total) return einval("need lo <= hi <= |Lambda|");
@@ -324,9 +331,9 @@ mf_status mf_search_range(mf_ctx* ctx, uint64_t lo, uint64_t hi, int32_t k, uint
   if (chunk > (1ull << 31)) chunk = 1ull << 31;
   DeviceGuard guard(ctx->device);
   cudaStream_t s = (cudaStream_t)stream;
-  const bool tc = ctx->precision == MF_BF16;
+  const bool tc = !fc && ctx->precision == MF_BF16;
   const int kcap = tc ? (k * 8 > 256 ? k * 8 : 256) : k;
-  const int grid = tc ? tc_grid(ctx) : f32_grid(ctx);
+  const int grid = fc ? fc_grid(ctx) : tc ? tc_grid(ctx) : f32_grid(ctx);
 
   // scratch: per-CTA lists, two merge buffers, merged list, rescored shortlist, count
   const size_t entries = (size_t)grid * kcap;
@@ -372,7 +379,7 @@ mf_status mf_search_range(mf_ctx* ctx, uint64_t lo, uint64_t hi, int32_t k, uint
     a.base = lo;
     a.len = 0;
     int nl = 1;
-    st = tc ? tc_search_chunk(ctx, a, s, &nl) : f32_search_chunk(ctx, a, s);
+    st = fc ? fc_search_chunk(ctx, a, s) : tc ? tc_search_chunk(ctx, a, s, &nl) : f32_search_chunk(ctx, a, s);
     if (st != MF_OK) return st;
     launches += nl;
     score_launches += nl;
@@ -381,7 +388,7 @@ mf_status mf_search_range(mf_ctx* ctx, uint64_t lo, uint64_t hi, int32_t k, uint
     a.base = b;
     a.len = (hi - b) < chunk ? (hi - b) : chunk;
     int nl = 1;
-    st = tc ? tc_search_chunk(ctx, a, s, &nl) : f32_search_chunk(ctx, a, s);
+    st = fc ? fc_search_chunk(ctx, a, s) : tc ? tc_search_chunk(ctx, a, s, &nl) : f32_search_chunk(ctx, a, s);
     if (st != MF_OK) return st;
     a.first = 0;
     launches += nl;

@@ -217,6 +217,9 @@ struct mf_ctx {
   void* d_tc = nullptr;           // packed bf16 operand images (tensor-core path)
   void* d_partial = nullptr;      // per-candidate partial objective between tensor-core passes
   size_t partial_bytes = 0;
+  // fixed-context mode: the per-option table of the last mf_fc_set
+  void* d_fc = nullptr;           // see mf::FcLayout
+  int fc_ready = 0;
   size_t tc_bytes = 0;
   mf::TcArgs tc{};
   // growable scratch (search lists, merge buffers, shortlist)
@@ -247,6 +250,18 @@ namespace mf {
 
 // Thread-local detail string of the last failure.
 void set_error(const std::string& msg);
+
+// Makes the context's device current for the scope of an API call.
+struct DeviceGuard {
+  int prev = -1;
+  bool changed = false;
+  explicit DeviceGuard(int dev) {
+    if (cudaGetDevice(&prev) == cudaSuccess && prev != dev) changed = cudaSetDevice(dev) == cudaSuccess;
+  }
+  ~DeviceGuard() {
+    if (changed) cudaSetDevice(prev);
+  }
+};
 mf_status cuda_fail(cudaError_t e, const char* what);
 
 #define MF_CUDA(call)                                         \
@@ -273,6 +288,10 @@ size_t f32_smem_bytes(const Params& P, int k, bool& resident);
 int f32_grid(const mf_ctx* c);
 mf_status f32_prepare(mf_ctx* c);
 mf_status f32_search_chunk(mf_ctx* c, const RangeArgs& a, cudaStream_t s);
+// Fixed-context mode: one range launch of the table-lookup scan over the per-option
+// table of mf_fc_set.
+int fc_grid(const mf_ctx* c);
+mf_status fc_search_chunk(mf_ctx* c, const RangeArgs& a, cudaStream_t s);
 mf_status f32_search_chunk_params(const Params& P, int grid, const RangeArgs& a, cudaStream_t s);
 mf_status f32_score_list(mf_ctx* c, const uint64_t* idx, const int32_t* genes, uint64_t n,
                          float* score, uint8_t* feas, float* pred, cudaStream_t s);

@@ -24,7 +24,8 @@ EMPTY = (1 << 64) - 1
 _EXPORTS = ["mf_status_string", "mf_last_error", "mf_create", "mf_destroy", "mf_space_size",
             "mf_set_objective", "mf_score_batch", "mf_search_range", "mf_search_exhaustive",
             "mf_ga_generation", "mf_ga_init", "mf_ga_step", "mf_ga_run", "mf_check_device_status",
-            "mf_get_stats", "mf_search_exhaustive_noalloc"]
+            "mf_get_stats", "mf_search_exhaustive_noalloc", "mf_fc_set", "mf_fc_table", "mf_fc_search",
+            "mf_vram_feasible"]
 
 
 class MFError(RuntimeError):
@@ -61,6 +62,13 @@ class _GAParams(C.Structure):
                 ("mutation_p", C.c_double), ("elitism", C.c_int32)]
 
 
+class _FcParams(C.Structure):
+    _fields_ = [("obs", C.c_void_p), ("variant", C.c_void_p), ("quality", C.c_void_p),
+                ("f_min", C.c_void_p), ("f_max", C.c_void_p), ("omega", C.c_void_p), ("tau", C.c_void_p),
+                ("reload_cost", C.c_void_p), ("prev_variant", C.c_void_p),
+                ("alpha", C.c_float), ("beta", C.c_float), ("delta", C.c_float)]
+
+
 def _load() -> C.CDLL:
     if not os.path.exists(LIB_PATH):
         raise ImportError(f"{LIB_PATH} is missing: build it with paper_2609_02109_gb300.build.build()")
@@ -82,6 +90,10 @@ def _load() -> C.CDLL:
     lib.mf_check_device_status.argtypes = [vp, vp]
     lib.mf_get_stats.argtypes = [vp, C.POINTER(_Stats)]
     lib.mf_search_exhaustive_noalloc.argtypes = [C.POINTER(_Problem), i32, u64, C.POINTER(_Result), vp]
+    lib.mf_fc_set.argtypes = [vp, C.POINTER(_FcParams), vp]
+    lib.mf_fc_table.argtypes = [vp, vp, vp, vp, vp, vp]
+    lib.mf_fc_search.argtypes = [vp, u64, u64, i32, u64, C.POINTER(_Result), vp]
+    lib.mf_vram_feasible.argtypes = [vp, u64, u64, vp, u64, C.POINTER(u64), vp]
     for name in _EXPORTS[2:]:
         getattr(lib, name).restype = st
     return lib
@@ -263,6 +275,57 @@ class Context:
         _check(_lib.mf_ga_run(self._h, C.byref(g), int(seed), genome.ctypes.data, C.byref(fit),
                               _stream(self.device)), "mf_ga_run")
         return float(fit.value), genome
+
+    # -- fixed-context mode ---------------------------------------------------
+    def fc_set(self, fc: dict) -> None:
+        """Evaluate the local predictions under fc["obs"] and build the utility table."""
+        keep = {
+            "obs": np.ascontiguousarray(fc["obs"], dtype=np.float32),
+            "variant": np.ascontiguousarray(fc["variant"], dtype=np.int32),
+            "quality": np.ascontiguousarray(fc["quality"], dtype=np.float32),
+            "f_min": np.ascontiguousarray(fc["f_min"], dtype=np.float32),
+            "f_max": np.ascontiguousarray(fc["f_max"], dtype=np.float32),
+            "omega": np.ascontiguousarray(fc["omega"], dtype=np.float32),
+            "tau": np.ascontiguousarray(fc["tau"], dtype=np.float32),
+            "reload_cost": np.ascontiguousarray(fc["reload_cost"], dtype=np.float32),
+            "prev_variant": np.ascontiguousarray(fc["prev_variant"], dtype=np.int32),
+        }
+        p = _FcParams(*(keep[k].ctypes.data for k in ("obs", "variant", "quality", "f_min", "f_max", "omega",
+                                                       "tau", "reload_cost", "prev_variant")),
+                      float(fc["alpha"]), float(fc["beta"]), float(fc["delta"]))
+        _check(_lib.mf_fc_set(self._h, C.byref(p), _stream(self.device)), "mf_fc_set")
+
+    def fc_table(self):
+        """(fhat, f, u, ok) of every option row, as numpy arrays."""
+        rows = int(self._keep["n_options"].sum())
+        dev = f"cuda:{self.device}"
+        fhat, f, u = (torch.empty(rows, dtype=torch.float32, device=dev) for _ in range(3))
+        ok = torch.empty(rows, dtype=torch.uint8, device=dev)
+        _check(_lib.mf_fc_table(self._h, fhat.data_ptr(), f.data_ptr(), u.data_ptr(), ok.data_ptr(),
+                                _stream(self.device)), "mf_fc_table")
+        torch.cuda.current_stream(self.device).synchronize()
+        return fhat.cpu().numpy(), f.cpu().numpy(), u.cpu().numpy(), ok.cpu().numpy().astype(bool)
+
+    def fc_search(self, k: int, lo: int = 0, hi: int | None = None, chunk: int = 0) -> dict:
+        hi = self.space_size if hi is None else int(hi)
+        ti = np.empty(k, dtype=np.uint64)
+        ts = np.empty(k, dtype=np.float32)
+        r = _Result(0, 0.0, 0, k, ti.ctypes.data, ts.ctypes.data)
+        _check(_lib.mf_fc_search(self._h, int(lo), hi, int(k), int(chunk), C.byref(r), _stream(self.device)),
+               "mf_fc_search")
+        return dict(best_idx=int(r.best_idx), best_score=float(r.best_score), count=int(r.feasible_count),
+                    topk_idx=ti, topk_score=ts)
+
+    def vram_feasible(self, lo: int = 0, hi: int | None = None, cap: int | None = None):
+        """(count, device tensor of the first min(count, cap) VRAM-feasible indices)."""
+        hi = self.space_size if hi is None else int(hi)
+        cap = (hi - int(lo)) if cap is None else int(cap)
+        out = torch.empty(max(cap, 1), dtype=torch.int64, device=f"cuda:{self.device}")
+        cnt = C.c_uint64(0)
+        _check(_lib.mf_vram_feasible(self._h, int(lo), hi, out.data_ptr(), cap, C.byref(cnt),
+                                     _stream(self.device)), "mf_vram_feasible")
+        c = int(cnt.value)
+        return c, out[:min(c, cap)]
 
     def stats(self) -> dict:
         st = _Stats()
