@@ -230,6 +230,42 @@ def stress_throughput(mf, torch, device):
                          "flops_per_candidate": flops_per_candidate(prob), "peak_source": f"{src} bf16 sustained"}}
 
 
+def fixed_context_throughput(mf, torch, device):
+    """Fixed-context mode (observed state held fixed, Eq. 3 utility): table build and
+    the table-lookup exhaustive scan over the large and stress spaces."""
+    peaks, _ = _peaks()
+    sms = torch.cuda.get_device_properties(device).multi_processor_count
+    issue = sms * 4 * 32 * float(peaks.get("sm_max_mhz", 2070.0)) * 1e6  # lane-instructions/s
+    out = {}
+    stream = torch.cuda.current_stream(device)
+    for name, prob, seed in (("large", W.large(precision="fp32"), 3), ("stress", W.stress(precision="fp32"), 5)):
+        fc = W.fc_scenario(prob, seed)
+        n = int(np.prod(prob["n_options"].astype(np.float64)))
+        N = int(prob["n_options"].size)
+        with mf.Context(prob, device=device) as ctx:
+            t0 = time.perf_counter()
+            ctx.fc_set(fc)
+            set_ms = 1e3 * (time.perf_counter() - t0)
+            ctx.fc_search(32, chunk=1 << 30)
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            torch.cuda.synchronize(device)
+            e0.record(stream)
+            res = ctx.fc_search(32, chunk=1 << 30)
+            e1.record(stream)
+            e1.synchronize()
+            st = ctx.stats()
+        ms = e0.elapsed_time(e1)
+        ops = 3 * N * n / (st["score_ms_last"] / 1e3)  # N table loads and 2N adds per candidate
+        out[name] = {"candidates": n, "value": n / (ms / 1e3), "unit": UNIT, "ms": ms, "fc_set_ms": set_ms,
+                     "count": res["count"],
+                     "roofline": {"bound": "alu", "achieved": ops, "peak": issue, "unit": "lane-ops/s",
+                                  "frac": ops / issue,
+                                  "peak_source": f"{sms} SMs x 4 schedulers x 32 lanes x max SM clock",
+                                  "ops_per_candidate": 3 * N}}
+    return out
+
+
 def ga_latency(mf, torch, device, decisions_per_scenario):
     """p50/p99 of complete GA decisions (host call -> result on host) over 8 scenarios."""
     g = W.GA_PARAMS
@@ -356,6 +392,7 @@ def run_gpu(args):
                "how": "mf_create from host arrays + mf_search_exhaustive + mf_destroy, host wall clock, median"}
 
     stress = stress_throughput(mf, torch, device) if rank == 0 and not args.no_stress else None
+    fixed = fixed_context_throughput(mf, torch, device) if rank == 0 and not args.no_stress else None
     ga = ga_latency(mf, torch, device, args.ga_decisions) if rank == 0 else None
     base = cpu_baseline(W.large(precision="fp32")) if (rank == 0 and world == 1 and not args.no_cpu) else None
     if rank == 0:
@@ -366,7 +403,7 @@ def run_gpu(args):
                 "cpu_baseline": base, "e2e": e2e, "gpu_launches": launches, "clocks": clk.summary(),
                 "feasible_fraction": feasible_frac, "best": {"idx": res["best_idx"], "J": res["best_score"],
                                                              "count": res["count"]},
-                "ga": ga, "stress": stress}
+                "ga": ga, "stress": stress, "fixed_context": fixed}
         print(json.dumps(line), flush=True)
     if dist:
         dist.barrier()

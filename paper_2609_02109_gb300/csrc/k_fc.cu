@@ -139,14 +139,19 @@ k_fc_local(const Params P, const FcLayout L, const FcConst C) {
 }
 
 // ---------------------------------------------------------------------------
-// Table-lookup scan: one candidate per thread and step; digits advance by the grid
-// stride with carries.  Per-CTA running top-k as in the fp32 scorer.
+// Table-lookup scan.  A step of the CTA covers 512 x kFcRun consecutive candidates:
+// thread t takes the run of kFcRun consecutive indices starting at step base + t *
+// kFcRun, so between them only the last model's option advances (the partial sum
+// over the other models is reused until a carry).  J is summed in model order
+// either way.  Per-CTA running top-k as in the fp32 scorer, one merge check per
+// step with a queue of one entry per candidate of the step.
 // ---------------------------------------------------------------------------
 constexpr int kFcThreads = 512;
+constexpr int kFcRun = 8;
 
 struct FcScan {
   const float2* tab;
-  uint32_t step[MF_MAX_MODELS];  // mixed-radix digits of the grid stride (grid x threads)
+  uint32_t step[MF_MAX_MODELS];  // mixed-radix digits of the grid step (grid x threads x kFcRun)
 };
 
 __global__ void __launch_bounds__(kFcThreads, 1)
@@ -154,16 +159,17 @@ k_fc_scan(const Params P, const FcScan S, const RangeArgs R) {
   extern __shared__ __align__(16) unsigned char sm[];
   const int N = P.n_models;
   const int sumK = pick(P.off, N - 1) + pick(P.K, N - 1);
+  constexpr int QCAP = kFcThreads * kFcRun;
   float2* tab = reinterpret_cast<float2*>(sm);
   unsigned char* q = sm + (((size_t)sumK * sizeof(float2) + 15) & ~(size_t)15);
   const int tid = threadIdx.x;
   CtaTopK tk;
   tk.li = reinterpret_cast<uint64_t*>(q); q += sizeof(uint64_t) * R.k;
   tk.ni = reinterpret_cast<uint64_t*>(q); q += sizeof(uint64_t) * R.k;
-  tk.qi = reinterpret_cast<uint64_t*>(q); q += sizeof(uint64_t) * kFcThreads;
+  tk.qi = reinterpret_cast<uint64_t*>(q); q += sizeof(uint64_t) * QCAP;
   tk.ls = reinterpret_cast<float*>(q); q += sizeof(float) * R.k;
   tk.ns = reinterpret_cast<float*>(q); q += sizeof(float) * R.k;
-  tk.qs = reinterpret_cast<float*>(q); q += sizeof(float) * kFcThreads;
+  tk.qs = reinterpret_cast<float*>(q); q += sizeof(float) * QCAP;
   tk.qn = reinterpret_cast<int*>(q);
   tk.k = R.k;
   for (int e = tid; e < sumK; e += blockDim.x) tab[e] = S.tab[e];
@@ -173,58 +179,87 @@ k_fc_scan(const Params P, const FcScan S, const RangeArgs R) {
     tk.li[e] = R.first ? kEmptyIdx : R.lists_i[gl + e];
   }
   if (tid == 0) *tk.qn = 0;
-  // this thread's first candidate and its option rows
-  const uint64_t t0 = (uint64_t)blockIdx.x * blockDim.x + tid;
-  int row[MF_MAX_MODELS];
+  // digits of this thread's first run start
+  const uint64_t t0 = ((uint64_t)blockIdx.x * blockDim.x + tid) * kFcRun;
+  int start[MF_MAX_MODELS];
   {
     const uint64_t idx0 = R.base + (t0 < R.len ? t0 : 0);
 #pragma unroll
     for (int i = 0; i < MF_MAX_MODELS; ++i)
-      if (i < N) row[i] = pick(P.off, i) + (int)((idx0 / pick(P.stride, i)) % (uint64_t)pick(P.K, i));
+      if (i < N) start[i] = P.off[i] + (int)((idx0 / P.stride[i]) % (uint64_t)P.K[i]);
   }
   __syncthreads();
   float thr_s = tk.ls[R.k - 1];
   uint64_t thr_i = tk.li[R.k - 1];
   const float cap = P.vram_cap;
+  const int last = N - 1;
+  const int off_last = pick(P.off, last);
+  const int end_last = off_last + pick(P.K, last);
   unsigned int my_count = 0;
-  const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
-  for (uint64_t base = (uint64_t)blockIdx.x * blockDim.x; base < R.len; base += stride) {
-    const uint64_t t = base + tid;
-    const bool valid = t < R.len;
-    float J = 0.f, V = 0.f;
+  const uint64_t gstep = (uint64_t)gridDim.x * blockDim.x * kFcRun;
+  for (uint64_t base = (uint64_t)blockIdx.x * blockDim.x * kFcRun; base < R.len; base += gstep) {
+    // the run: rows from `start`, the prefix sum over models 0..N-2 until a carry
+    int row[MF_MAX_MODELS];
+#pragma unroll
+    for (int i = 0; i < MF_MAX_MODELS; ++i) row[i] = start[i];
+    float pJ = 0.f, pV = 0.f;
 #pragma unroll
     for (int i = 0; i < MF_MAX_MODELS; ++i)
-      if (i < N) {
-        const float2 e = tab[row[i]];
-        J += e.x;
-        V += e.y;
+      if (i < last) { const float2 e = tab[row[i]]; pJ += e.x; pV += e.y; }
+    int rl = pick(row, last);
+    bool any = false;
+    const uint64_t t1 = base + (uint64_t)tid * kFcRun;
+#pragma unroll
+    for (int u = 0; u < kFcRun; ++u) {
+      const uint64_t t = t1 + u;
+      const float2 e = tab[rl];
+      const float J = pJ + e.x, V = pV + e.y;
+      // -inf below a floor; NaN compares false
+      const bool feas = t < R.len && V <= cap && J > -INFINITY;
+      const uint64_t idx = R.base + t;
+      my_count += feas ? 1u : 0u;
+      if (feas && precedes(J, idx, thr_s, thr_i)) {
+        const int pos = atomicAdd(tk.qn, 1);
+        tk.qs[pos] = J;
+        tk.qi[pos] = idx;
+        any = true;
       }
-    // -inf below a floor; NaN compares false
-    const bool feas = valid && V <= cap && J > -INFINITY;
-    const uint64_t idx = R.base + t;
-    my_count += feas ? 1u : 0u;
-    const bool push = feas && precedes(J, idx, thr_s, thr_i);
-    if (push) {
-      const int pos = atomicAdd(tk.qn, 1);
-      tk.qs[pos] = J;
-      tk.qi[pos] = idx;
+      // next index: the last model's option, with a carry into the prefix
+      if (++rl == end_last) {
+        rl = off_last;
+        bool carry = true;
+#pragma unroll
+        for (int i = MF_MAX_MODELS - 1; i >= 0; --i)
+          if (i < last && carry) {
+            const int off = P.off[i];
+            int d = row[i] - off + 1;
+            carry = d == P.K[i];
+            if (carry) d = 0;
+            row[i] = off + d;
+          }
+        pJ = 0.f;
+        pV = 0.f;
+#pragma unroll
+        for (int i = 0; i < MF_MAX_MODELS; ++i)
+          if (i < last) { const float2 e2 = tab[row[i]]; pJ += e2.x; pV += e2.y; }
+      }
     }
-    if (__syncthreads_or(push)) {  // block-uniform
+    if (__syncthreads_or(any)) {  // block-uniform
       topk_merge(tk, tid, blockDim.x, [] __device__() { __syncthreads(); });
       thr_s = tk.ls[R.k - 1];
       thr_i = tk.li[R.k - 1];
     }
-    // advance the digits by the stride, last model first
+    // advance the run start by the grid step, last model first
     uint32_t carry = 0;
 #pragma unroll
     for (int i = MF_MAX_MODELS - 1; i >= 0; --i)
       if (i < N) {
-        const int off = pick(P.off, i);
-        const uint32_t K = (uint32_t)pick(P.K, i);
-        uint32_t d = (uint32_t)(row[i] - off) + S.step[i] + carry;
+        const int off = P.off[i];
+        const uint32_t K = (uint32_t)P.K[i];
+        uint32_t d = (uint32_t)(start[i] - off) + S.step[i] + carry;
         carry = d >= K;
         if (carry) d -= K;
-        row[i] = off + (int)d;
+        start[i] = off + (int)d;
       }
   }
   for (int e = tid; e < R.k; e += blockDim.x) {
@@ -269,7 +304,7 @@ k_vram(const Params P, const VramArgs A) {
     const uint64_t idx0 = A.lo + (s0 + tid < A.len ? s0 + tid : 0);
 #pragma unroll
     for (int i = 0; i < MF_MAX_MODELS; ++i)
-      if (i < N) row[i] = pick(P.off, i) + (int)((idx0 / pick(P.stride, i)) % (uint64_t)pick(P.K, i));
+      if (i < N) row[i] = P.off[i] + (int)((idx0 / P.stride[i]) % (uint64_t)P.K[i]);
   }
   if (tid == 0) s_base = WRITE ? A.counts[blockIdx.x] : 0ull;
   __syncthreads();
@@ -303,8 +338,8 @@ k_vram(const Params P, const VramArgs A) {
 #pragma unroll
     for (int i = MF_MAX_MODELS - 1; i >= 0; --i)
       if (i < N) {
-        const int off = pick(P.off, i);
-        const uint32_t K = (uint32_t)pick(P.K, i);
+        const int off = P.off[i];
+        const uint32_t K = (uint32_t)P.K[i];
         uint32_t d = (uint32_t)(row[i] - off) + A.step[i] + carry;
         carry = d >= K;
         if (carry) d -= K;
@@ -352,9 +387,9 @@ mf_status fc_search_chunk(mf_ctx* c, const RangeArgs& a, cudaStream_t s) {
   fc_bytes(c->sumK, c->P.n_models, &L, (char*)c->d_fc);
   FcScan S{};
   S.tab = L.tab;
-  radix_digits(c->P, (uint64_t)fc_grid(c) * kFcThreads, S.step);
+  radix_digits(c->P, (uint64_t)fc_grid(c) * kFcThreads * kFcRun, S.step);
   const size_t smem = (((size_t)c->sumK * sizeof(float2) + 15) & ~(size_t)15) +
-                      (sizeof(uint64_t) + sizeof(float)) * (2 * (size_t)a.k + kFcThreads) + 16;
+                      (sizeof(uint64_t) + sizeof(float)) * (2 * (size_t)a.k + kFcThreads * kFcRun) + 16;
   if (smem > 227 * 1024) {
     set_error("fixed-context search: top-k lists do not fit shared memory; use a smaller k");
     return MF_EUNSUPPORTED;
