@@ -550,3 +550,123 @@ uint64_t orc_vram_feasible(const orc_problem *p, uint64_t lo, uint64_t hi, uint6
   }
   return c;
 }
+
+/* ---------------------------------------------------------------------------
+ * Eq. 3 utility on the coupled aggregate (the predictors see the candidate's own
+ * summed demands, as in orc_score_digits).
+ * ------------------------------------------------------------------------- */
+
+/* Model i's term of Eq. 3 from its raw predicted throughput fhat (option row r). */
+static double util_term(const orc_fc *fc, int32_t i, int64_t r, double fhat, int32_t *ok) {
+  const double f = (fhat - (double)fc->f_min[r]) / ((double)fc->f_max[r] - (double)fc->f_min[r]);
+  const int32_t eta = fc->prev_variant[i] >= 0 && fc->variant[r] != fc->prev_variant[i];
+  const double margin = (double)fc->tau[i] + (double)fc->delta - f;
+  *ok = f >= (double)fc->tau[i];
+  return (double)fc->omega[i] * f * (double)fc->quality[r] -
+         (double)fc->alpha * (double)eta * (double)fc->reload_cost[i] -
+         (double)fc->beta * (margin > 0.0 ? margin * margin : 0.0);
+}
+
+double orc_util_score_digits(const orc_problem *p, const orc_fc *fc, const int32_t *o, int32_t *feasible,
+                             double *pred, double *agg) {
+  const int32_t n = p->n_models, dl = p->d_local, din = d_in_of(p);
+  double A[4] = {0.0, 0.0, 0.0, (double)n};
+  for (int32_t i = 0; i < n; ++i) {
+    const float *d = p->demand + 3 * (option_offset(p, i) + o[i]);
+    A[0] += (double)d[0];
+    A[1] += (double)d[1];
+    A[2] += (double)d[2];
+  }
+  double s[4];
+  if (p->agg_scale) {
+    for (int c = 0; c < 4; ++c) s[c] = (double)p->agg_scale[c];
+  } else {
+    s[0] = 1.0 / (0.6 * n); s[1] = 1.0 / (20.0 * n); s[2] = 1.0 / (1500.0 * n); s[3] = 1.0 / 8.0;
+    for (int c = 0; c < 4; ++c) s[c] = (double)(float)s[c];
+  }
+  if (agg) for (int c = 0; c < 4; ++c) agg[c] = A[c];
+  double z[din];
+  double J = 0.0;
+  int32_t floors = 1;
+  for (int32_t i = 0; i < n; ++i) {
+    const int64_t r = option_offset(p, i) + o[i];
+    const float *x = p->local_feats + (int64_t)dl * r;
+    for (int32_t k = 0; k < dl; ++k) z[k] = (double)x[k];
+    for (int c = 0; c < 4; ++c) z[dl + c] = A[c] * s[c];
+    double thr, lat;
+    predictor(p, i, z, &thr, &lat, NULL);
+    if (pred) { pred[2 * i] = thr; pred[2 * i + 1] = lat; }
+    int32_t ok;
+    J += util_term(fc, i, r, thr, &ok);
+    floors = floors && ok;
+  }
+  int32_t feas = floors && A[1] <= (double)p->vram_cap;
+  if (isnan(J)) feas = 0;
+  if (feasible) *feasible = feas;
+  return feas ? J : -INFINITY;
+}
+
+void orc_util_score_list(const orc_problem *p, const orc_fc *fc, const uint64_t *idx, uint64_t n,
+                         double *score, int32_t *feasible, double *pred, double *agg, int32_t nthreads) {
+  const uint64_t size = orc_space_size(p);
+  const int32_t N = p->n_models;
+  if (nthreads < 1) nthreads = 1;
+#ifdef _OPENMP
+#pragma omp parallel for num_threads(nthreads) schedule(static)
+#endif
+  for (int64_t t = 0; t < (int64_t)n; ++t) {
+    int32_t o[64];
+    int32_t f = 0;
+    double J = -INFINITY;
+    if (idx[t] < size) {
+      orc_decode(p, idx[t], o);
+      J = orc_util_score_digits(p, fc, o, &f, pred ? pred + 2 * N * t : NULL, agg ? agg + 4 * t : NULL);
+    } else if (pred) {
+      for (int32_t j = 0; j < 2 * N; ++j) pred[2 * N * t + j] = NAN;
+    }
+    score[t] = J;
+    if (feasible) feasible[t] = f;
+  }
+}
+
+void orc_util_exhaustive(const orc_problem *p, const orc_fc *fc, uint64_t lo, uint64_t hi, int32_t k,
+                         uint64_t *topk_idx, double *topk_score, uint64_t *count, int32_t nthreads) {
+  for (int32_t j = 0; j < k; ++j) { topk_idx[j] = UINT64_MAX; topk_score[j] = -INFINITY; }
+  uint64_t total_count = 0;
+  const uint64_t size = orc_space_size(p);
+  if (hi > size) hi = size;
+  if (nthreads < 1) nthreads = 1;
+#ifdef _OPENMP
+#pragma omp parallel num_threads(nthreads)
+#endif
+  {
+    uint64_t *li = (uint64_t *)malloc(sizeof(uint64_t) * (size_t)k);
+    double *ls = (double *)malloc(sizeof(double) * (size_t)k);
+    for (int32_t j = 0; j < k; ++j) { li[j] = UINT64_MAX; ls[j] = -INFINITY; }
+    uint64_t c = 0;
+    int32_t o[64];
+#ifdef _OPENMP
+#pragma omp for schedule(dynamic, 4096)
+#endif
+    for (int64_t t = (int64_t)lo; t < (int64_t)hi; ++t) {
+      int32_t f = 0;
+      orc_decode(p, (uint64_t)t, o);
+      const double J = orc_util_score_digits(p, fc, o, &f, NULL, NULL);
+      if (f) {
+        ++c;
+        topk_insert(k, li, ls, J, (uint64_t)t);
+      }
+    }
+#ifdef _OPENMP
+#pragma omp critical
+#endif
+    {
+      total_count += c;
+      for (int32_t j = 0; j < k; ++j)
+        if (li[j] != UINT64_MAX) topk_insert(k, topk_idx, topk_score, ls[j], li[j]);
+    }
+    free(li);
+    free(ls);
+  }
+  *count = total_count;
+}

@@ -23,6 +23,9 @@
  *                                     reload term = alpha c, quadratic margin term,
  *                                     linear case as one matrix product)
  *   orc_vram_feasible                 pinned (two-pointer count, brute-force list)
+ *   orc_util_*                        pinned (hand example, equal to the fixed-context
+ *                                     utility when the aggregate is unused, reduces to
+ *                                     the weighted-throughput objective)
  */
 #ifndef MF_ORACLE_H
 #define MF_ORACLE_H
@@ -132,6 +135,19 @@ double orc_fc_score_digits(const orc_problem *p, const orc_fc *fc, const int32_t
  * the feasible count; unfilled slots are (UINT64_MAX, -inf). */
 void orc_fc_exhaustive(const orc_problem *p, const orc_fc *fc, uint64_t lo, uint64_t hi, int32_t k,
                        uint64_t *topk_idx, double *topk_score, uint64_t *count, int32_t nthreads);
+
+/* ---------------------------------------------------------------------------
+ * The Eq. 3 utility on the coupled aggregate: each predictor sees the candidate's
+ * own summed demands (as orc_score_digits) and its throughput output enters Eq. 3
+ * through the per-option terms of orc_fc (obs is not used).  Constraints: Eq. 4
+ * floors f_i >= tau_i and the VRAM bound.
+ * ------------------------------------------------------------------------- */
+double orc_util_score_digits(const orc_problem *p, const orc_fc *fc, const int32_t *o, int32_t *feasible,
+                             double *pred, double *agg);
+void orc_util_score_list(const orc_problem *p, const orc_fc *fc, const uint64_t *idx, uint64_t n,
+                         double *score, int32_t *feasible, double *pred, double *agg, int32_t nthreads);
+void orc_util_exhaustive(const orc_problem *p, const orc_fc *fc, uint64_t lo, uint64_t hi, int32_t k,
+                         uint64_t *topk_idx, double *topk_score, uint64_t *count, int32_t nthreads);
 
 /* The VRAM-feasible joint configurations in [lo, hi) (Lambda with the
  * VRAM-infeasible configurations removed), ascending; writes at most cap of

@@ -91,6 +91,11 @@ def _load():
             lib.orc_fc_exhaustive.argtypes = [P, F, u64, u64, i32, vp, vp, vp, i32]
             lib.orc_fc_exhaustive.restype = None
             lib.orc_vram_feasible.argtypes = [P, u64, u64, vp, u64]; lib.orc_vram_feasible.restype = u64
+            lib.orc_util_score_digits.argtypes = [P, F, vp, vp, vp, vp]; lib.orc_util_score_digits.restype = dbl
+            lib.orc_util_score_list.argtypes = [P, F, vp, u64, vp, vp, vp, vp, i32]
+            lib.orc_util_score_list.restype = None
+            lib.orc_util_exhaustive.argtypes = [P, F, u64, u64, i32, vp, vp, vp, i32]
+            lib.orc_util_exhaustive.restype = None
             _lib = lib
     return _lib
 
@@ -242,6 +247,39 @@ class Oracle:
         cnt = np.zeros(1, dtype=np.uint64)
         self.lib.orc_fc_exhaustive(C.byref(self.p), C.byref(f_), int(lo), hi, int(k), _ptr(ti), _ptr(ts),
                                    _ptr(cnt), self.nthreads)
+        return ti, ts, int(cnt[0])
+
+    # -- Eq. 3 utility on the coupled aggregate -----------------------------------
+    def util_score_digits(self, fc: dict, digits):
+        f_ = self._fc(fc)
+        o = np.ascontiguousarray(digits, dtype=np.int32)
+        feas = np.zeros(1, dtype=np.int32)
+        pred = np.empty((self.n, 2))
+        J = self.lib.orc_util_score_digits(C.byref(self.p), C.byref(f_), _ptr(o), _ptr(feas), _ptr(pred), None)
+        return float(J), bool(feas[0]), pred
+
+    def util_score_list(self, fc: dict, idx, with_pred: bool = False):
+        f_ = self._fc(fc)
+        idx = np.ascontiguousarray(idx, dtype=np.uint64)
+        n = idx.size
+        score = np.empty(n)
+        feas = np.empty(n, dtype=np.int32)
+        pred = np.empty((n, self.n, 2)) if with_pred else None
+        agg = np.empty((n, 4)) if with_pred else None
+        self.lib.orc_util_score_list(C.byref(self.p), C.byref(f_), _ptr(idx), n, _ptr(score), _ptr(feas),
+                                     _ptr(pred), _ptr(agg), self.nthreads)
+        if with_pred:
+            return score, feas.astype(bool), pred, agg
+        return score, feas.astype(bool)
+
+    def util_exhaustive(self, fc: dict, k: int, lo: int = 0, hi: int | None = None):
+        f_ = self._fc(fc)
+        hi = self.space_size() if hi is None else int(hi)
+        ti = np.empty(k, dtype=np.uint64)
+        ts = np.empty(k, dtype=np.float64)
+        cnt = np.zeros(1, dtype=np.uint64)
+        self.lib.orc_util_exhaustive(C.byref(self.p), C.byref(f_), int(lo), hi, int(k), _ptr(ti), _ptr(ts),
+                                     _ptr(cnt), self.nthreads)
         return ti, ts, int(cnt[0])
 
     def vram_feasible(self, lo: int = 0, hi: int | None = None, cap: int | None = None):

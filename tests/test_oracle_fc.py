@@ -156,3 +156,65 @@ def test_vram_feasible_list_matches_two_pointer_count(oracle_mod):
     assert np.array_equal(lst, idx[ok].astype(np.uint64))
     c2, lst2 = o.vram_feasible(50, 150, cap=10)
     assert c2 == int(ok[50:150].sum()) and np.array_equal(lst2, idx[50:150][ok[50:150]][:10].astype(np.uint64))
+
+
+# ---------------------------------------------------------------------------
+# The Eq. 3 utility on the coupled aggregate (the predictors see the candidate's
+# own summed demands)
+# ---------------------------------------------------------------------------
+
+def test_util_hand_example(oracle_mod):
+    """The hand example's coupled aggregate of (0, 1) is (0.5 SM, 20 GB, ...), the
+    observed state of the fixed-context hand example, so J(1) = 0.54 again; (0, 0)
+    (aggregate 0.3 SM, 10 GB) and (1, 0) (0.5 SM, 16 GB) leave model B at f = 0 below
+    its floor, (1, 1) exceeds 24 GB."""
+    o = oracle_mod.Oracle(W.hand_example())
+    fc = _hand_fc()
+    J, f, pred = o.util_score_digits(fc, [0, 1])
+    assert f and abs(J - 0.54) < 1e-6
+    np.testing.assert_allclose(pred[:, 0], [0.6, 0.25], atol=1e-6)
+    J0, f0, p0 = o.util_score_digits(fc, [0, 0])
+    assert not f0 and J0 == -np.inf
+    np.testing.assert_allclose(p0[:, 0], [0.8, 0.0], atol=1e-6)  # A: 2 relu(0.5 - 0.1), B: relu(0.25 - 0.3)
+    J2, f2, p2 = o.util_score_digits(fc, [1, 0])
+    assert not f2 and abs(p2[0, 0] - 1.68) < 1e-6
+    ti, ts, cnt = o.util_exhaustive(fc, 4)
+    assert cnt == 1 and int(ti[0]) == 1 and abs(ts[0] - 0.54) < 1e-6
+
+
+def test_util_equals_fixed_context_when_the_aggregate_is_unused(oracle_mod):
+    """With W1's aggregate columns zero, the coupled utility cannot see the aggregate,
+    so it equals the fixed-context utility under any observed state."""
+    prob = W.make_problem([4, 3, 5], 8, 32, 16, 9, 30.0)
+    per = W.param_count(8, 32, 16)
+    w = prob["weights"].copy()
+    for i in range(3):
+        W1 = w[i * per:i * per + 32 * 12].reshape(32, 12)
+        W1[:, 8:] = 0.0
+    prob["weights"] = w
+    fc = W.fc_scenario(prob, 6)
+    o = oracle_mod.Oracle(prob)
+    for obs in (fc["obs"], np.array([9.0, 1.0, 123.0, 3.0], np.float32)):
+        f2 = dict(fc, obs=obs)
+        a = o.util_exhaustive(f2, 16)
+        b = o.fc_exhaustive(f2, 16)
+        assert a[2] == b[2] and 0 < a[2] < o.space_size()
+        assert np.array_equal(a[0], b[0])
+        np.testing.assert_allclose(a[1], b[1], rtol=1e-12)
+
+
+def test_util_reduces_to_weighted_throughput(oracle_mod):
+    """f_min = 0, f_max = 1, Q = 1, alpha = beta = 0, omega = w and floors far below:
+    J = sum_i w_i thr_i, the weighted-throughput objective with the SLA switched off."""
+    prob = W.paper_scale()
+    rows = int(prob["n_options"].sum())
+    fc = dict(W.fc_scenario(prob, 3), f_min=np.zeros(rows, np.float32), f_max=np.ones(rows, np.float32),
+              quality=np.ones(rows, np.float32), alpha=0.0, beta=0.0, omega=prob["obj_w"],
+              tau=np.full(5, -1e30, np.float32))
+    ref = dict(prob, sla=np.full(5, 1e30, np.float32))
+    o, r = oracle_mod.Oracle(prob), oracle_mod.Oracle(ref)
+    idx = np.random.default_rng(2).integers(0, o.space_size(), 500).astype(np.uint64)
+    a, fa = o.util_score_list(fc, idx)
+    b, fb = r.score_list(idx)
+    assert np.array_equal(fa, fb) and fa.all()
+    np.testing.assert_allclose(a, b, rtol=1e-12, atol=1e-15)
