@@ -54,7 +54,8 @@ typedef enum {
 } mf_status;
 
 typedef enum { MF_FP32 = 0, MF_BF16 = 1 } mf_precision;
-typedef enum { MF_OBJ_WEIGHTED_THR = 0, MF_OBJ_SOFT_LAT = 1 } mf_objective;
+/* MF_OBJ_UTILITY (Eq. 3 utility with floors) is set with mf_set_utility only. */
+typedef enum { MF_OBJ_WEIGHTED_THR = 0, MF_OBJ_SOFT_LAT = 1, MF_OBJ_UTILITY = 2 } mf_objective;
 typedef enum { MF_ACT_IDENTITY = 0, MF_ACT_SIGMOID = 1 } mf_out_act;
 
 #define MF_MAX_MODELS 16
@@ -259,6 +260,17 @@ mf_status mf_fc_search(mf_ctx *ctx, uint64_t lo, uint64_t hi, int32_t k, uint64_
  * their number to *count (host).  Synchronous. */
 mf_status mf_vram_feasible(mf_ctx *ctx, uint64_t lo, uint64_t hi, uint64_t *d_out, uint64_t cap,
                            uint64_t *count, void *stream);
+
+/* Score with the Eq. 3 utility on the coupled aggregate: predictor i sees the
+ * candidate's own summed demands (as every other call of this library) and its
+ * throughput output fhat_i enters J = sum_i [omega_i f_i Q_i - alpha eta_i c_i -
+ * beta max(0, tau_i + delta - f_i)^2], f_i = (fhat_i - f_min) / (f_max - f_min) of
+ * the option's variant; a candidate is feasible iff its summed VRAM <= vram_cap and
+ * f_i >= tau_i for every model (the latency outputs and SLA ceilings are not used).
+ * Applies to mf_score_batch, mf_search_range / mf_search_exhaustive (fp32 and bf16),
+ * mf_ga_generation and mf_ga_run until mf_set_utility(ctx, NULL) restores the
+ * problem's own objective.  p->obs is not used.  MF_EINVAL as mf_fc_set. */
+mf_status mf_set_utility(mf_ctx *ctx, const mf_fc_params *p);
 
 /* Read the context's instrumentation (see mf_stats). */
 mf_status mf_get_stats(const mf_ctx *ctx, mf_stats *out);

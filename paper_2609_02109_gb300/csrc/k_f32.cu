@@ -261,7 +261,7 @@ k_score_f32(const Params P, const RangeArgs R, const ListArgs L) {
           L.pred[(t * N + i) * 2 + 0] = thr;
           L.pred[(t * N + i) * 2 + 1] = lat;
         }
-        acc.add(P, i, thr, lat);
+        acc.add(P, i, thr, lat, row);
       }
       feas = acc.finish(P, A1);
     } else {
@@ -461,7 +461,10 @@ __global__ void k_combine(const Params P, const uint64_t* __restrict__ idx,
   if (ok) {
     Acc acc;
     acc.init();
-    for (int i = 0; i < N; ++i) acc.add(P, i, pred[(t * N + i) * 2], pred[(t * N + i) * 2 + 1]);
+    for (int i = 0; i < N; ++i) {
+      const int o = genes ? genes[t * N + i] : digit_of(P, id, i);
+      acc.add(P, i, pred[(t * N + i) * 2], pred[(t * N + i) * 2 + 1], P.off[i] + o);
+    }
     f = acc.finish(P, A1);
     J = acc.J;
   }

@@ -459,7 +459,8 @@ k_ga_persist(const Params P, const GaArgs g, const GaPersist G) {
   }
   // per-lane constants of model `lane`
   float my_w = 0.f, my_sla = 0.f, my_b3t = 0.f, my_b3l = 0.f;
-  int my_off = 0, my_K = 1;
+  float my_uomega = 0.f, my_utau = 0.f, my_ucost = 0.f;
+  int my_off = 0, my_K = 1, my_uprev = -1;
   if (lane < N) {
     const float* b3 = P.w32 + (size_t)lane * P.per_model + H * DIN + H + H * H + H + 2 * H;
     my_b3t = __ldg(b3);
@@ -468,6 +469,10 @@ k_ga_persist(const Params P, const GaArgs g, const GaPersist G) {
     my_sla = pick(P.sla, lane);
     my_off = pick(P.off, lane);
     my_K = pick(P.K, lane);
+    my_uomega = pick(P.u_omega, lane);
+    my_utau = pick(P.u_tau, lane);
+    my_ucost = pick(P.u_cost, lane);
+    my_uprev = pick(P.u_prev, lane);
   }
   for (int e = tid; e < N * SM * H; e += blockDim.x) sh1[e] = 0.f;
   for (int e = tid; e < sumK * DL; e += blockDim.x) sx[e] = P.x[e];
@@ -607,10 +612,17 @@ k_ga_persist(const Params P, const GaArgs g, const GaPersist G) {
         }
         t = out_act(P, t);
         l = out_act(P, l);
-        J = my_w * t;
-        ok = l <= my_sla;
-        const float over = l - my_sla;
-        pen = over > 0.f ? over : 0.f;
+        if (P.objective == MF_OBJ_UTILITY) {  // Eq. 3 utility, floor f >= tau
+          float f;
+          J = util_term_of(P, P.util[my_off + sgenes[warp * N + lane]], my_uomega, my_utau, my_ucost, my_uprev, t,
+                           &f);
+          ok = f >= my_utau;
+        } else {
+          J = my_w * t;
+          ok = l <= my_sla;
+          const float over = l - my_sla;
+          pen = over > 0.f ? over : 0.f;
+        }
       }
 #pragma unroll
       for (int o = 4; o > 0; o >>= 1) {  // lanes 0-7 hold the models
@@ -620,8 +632,8 @@ k_ga_persist(const Params P, const GaArgs g, const GaPersist G) {
       ok = __all_sync(0xffffffffu, ok);
       if (lane == 0) {
         bool feas = sagg[4 * warp + 3] <= P.vram_cap;
-        if (P.objective == MF_OBJ_WEIGHTED_THR) feas = feas && ok;
-        else J = fmaf(-P.soft_penalty, pen, J);
+        if (P.objective == MF_OBJ_SOFT_LAT) J = fmaf(-P.soft_penalty, pen, J);
+        else feas = feas && ok;
         if (J != J) feas = false;
         const float f = feas ? J : -INFINITY;
         st_word(&rec_cur[cg].fw, tagged(tag, __float_as_uint(f)));

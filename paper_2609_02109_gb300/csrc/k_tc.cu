@@ -211,8 +211,8 @@ __device__ __forceinline__ void mma_steps(int steps, uint32_t d_tmem, uint32_t a
 // KW: 32-bit words of an A1 row (8 or 16); AWO: word where the aggregate starts, or
 // -1 to take it from T at run time.  S1, S2, S3: K-steps of the three layers (0 = run time).
 // MP: the models run in several passes (T.m0..T.m1 and a partial record per candidate);
-// otherwise all N models in one launch.
-template <int MODE, int KW, int AWO, int S1, int S2, int S3, bool MP>
+// otherwise all N models in one launch.  UT: the Eq. 3 utility objective.
+template <int MODE, int KW, int AWO, int S1, int S2, int S3, bool MP, bool UT>
 __global__ void __launch_bounds__(kTcMaxPipes * 128, 1)
 k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   extern __shared__ __align__(1024) unsigned char smem[];
@@ -499,6 +499,14 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
         L.pred[(t * N + i) * 2 + 0] = thr;
         L.pred[(t * N + i) * 2 + 1] = lat;
       }
+      if (UT) {  // Eq. 3 utility, floors f >= tau
+        float f;
+        J += util_term(P, i, rows[i * 128 + row], thr, &f);
+        const float tau = P.u_tau[i];
+        sla_ok = sla_ok && (f >= tau);
+        sla_near = sla_near && (f >= tau - 2e-2f * fmaxf(fabsf(tau), fabsf(f)));
+        continue;
+      }
       J = fmaf(P.w[i], thr, J);
       const float sla = P.sla[i];
       sla_ok = sla_ok && (lat <= sla);
@@ -521,11 +529,11 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     }
     bool feas = valid && A1 <= vcap;
     bool cand = feas;
-    if (P.objective == MF_OBJ_WEIGHTED_THR) {
+    if (!UT && P.objective == MF_OBJ_SOFT_LAT) {
+      J = fmaf(-P.soft_penalty, pen, J);
+    } else {  // latency ceilings, or the utility's floors
       feas = feas && sla_ok;
       cand = cand && sla_near;
-    } else {
-      J = fmaf(-P.soft_penalty, pen, J);
     }
     if (J != J) { feas = false; cand = false; }
     if (MODE == kTcList) {
@@ -627,18 +635,24 @@ using TcFn = void (*)(const Params, const TcArgs, const RangeArgs, const TcList)
 
 // Instantiations: the two benchmark shapes (d_L 8, 64-64 and d_L 16, 128-128) with all
 // counts fixed at compile time, and a run-time fallback per A1 row width.
-template <int MODE, bool MP>
+template <int MODE, bool MP, bool UT>
 TcFn tc_kernel_mode(const TcArgs& T) {
   // S1 = k1 / 16, S2 = h1 / 16 + 1 (the b2 step), S3 = hl / 16
-  if (T.kw == 8 && T.dle == 8 && T.h1 == 64 && T.h2 == 64) return k_score_tc<MODE, 8, 4, 1, 5, 4, MP>;
-  if (T.kw == 16 && T.dle == 16 && T.h1 == 128 && T.h2 == 128) return k_score_tc<MODE, 16, 8, 2, 9, 8, MP>;
-  if (T.kw == 8) return k_score_tc<MODE, 8, -1, 0, 0, 0, MP>;
-  return k_score_tc<MODE, 16, -1, 0, 0, 0, MP>;
+  if (T.kw == 8 && T.dle == 8 && T.h1 == 64 && T.h2 == 64) return k_score_tc<MODE, 8, 4, 1, 5, 4, MP, UT>;
+  if (T.kw == 16 && T.dle == 16 && T.h1 == 128 && T.h2 == 128) return k_score_tc<MODE, 16, 8, 2, 9, 8, MP, UT>;
+  if (T.kw == 8) return k_score_tc<MODE, 8, -1, 0, 0, 0, MP, UT>;
+  return k_score_tc<MODE, 16, -1, 0, 0, 0, MP, UT>;
 }
 
-TcFn tc_kernel(int mode, const TcArgs& T) {
-  if (T.npasses > 1) return mode == kTcRange ? tc_kernel_mode<kTcRange, true>(T) : tc_kernel_mode<kTcList, true>(T);
-  return mode == kTcRange ? tc_kernel_mode<kTcRange, false>(T) : tc_kernel_mode<kTcList, false>(T);
+template <bool UT>
+TcFn tc_kernel_ut(int mode, const TcArgs& T) {
+  if (T.npasses > 1)
+    return mode == kTcRange ? tc_kernel_mode<kTcRange, true, UT>(T) : tc_kernel_mode<kTcList, true, UT>(T);
+  return mode == kTcRange ? tc_kernel_mode<kTcRange, false, UT>(T) : tc_kernel_mode<kTcList, false, UT>(T);
+}
+
+TcFn tc_kernel(int mode, const TcArgs& T, bool util) {
+  return util ? tc_kernel_ut<true>(mode, T) : tc_kernel_ut<false>(mode, T);
 }
 constexpr uint32_t kSmemFloor = 120 * 1024;          // keeps one CTA (one TMEM owner) per SM
 
@@ -810,8 +824,10 @@ mf_status tc_prepare(mf_ctx* c) {
   c->stats.h2d_bytes_create += img.size() + xw.size() * 4;
   T.img = base;
   T.xw = reinterpret_cast<const uint32_t*>(base + o_xw);
-  MF_CUDA(cudaFuncSetAttribute(tc_kernel(kTcRange, T), cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit));
-  MF_CUDA(cudaFuncSetAttribute(tc_kernel(kTcList, T), cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit));
+  for (int u = 0; u < 2; ++u) {
+    MF_CUDA(cudaFuncSetAttribute(tc_kernel(kTcRange, T, u), cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit));
+    MF_CUDA(cudaFuncSetAttribute(tc_kernel(kTcList, T, u), cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit));
+  }
   layout_smem(P, T, 0);
   if (T.sm_total > kSmemLimit) {
     set_error("tensor-core path: tables and weights exceed shared memory");
@@ -851,7 +867,7 @@ mf_status tc_search_chunk(mf_ctx* c, const RangeArgs& a, cudaStream_t s, int* nl
     r.first = a.first && b == 0;
     for (int p = 0; p < T.npasses; ++p) {
       set_pass(T, p, partial);
-      tc_kernel(kTcRange, T)<<<c->num_sms, T.pipes * 128, smem, s>>>(c->P, T, r, L);
+      tc_kernel(kTcRange, T, c->P.objective == MF_OBJ_UTILITY)<<<c->num_sms, T.pipes * 128, smem, s>>>(c->P, T, r, L);
       MF_CUDA(cudaGetLastError());
       ++launches;
     }
@@ -881,7 +897,7 @@ mf_status tc_score_list(mf_ctx* c, const uint64_t* idx, uint64_t n, float* score
     TcList L{idx + b, m, score + b, feas ? feas + b : nullptr, pred ? pred + b * N * 2 : nullptr};
     for (int p = 0; p < T.npasses; ++p) {
       set_pass(T, p, partial);
-      tc_kernel(kTcList, T)<<<(unsigned)grid, T.pipes * 128, smem, s>>>(c->P, T, R, L);
+      tc_kernel(kTcList, T, c->P.objective == MF_OBJ_UTILITY)<<<(unsigned)grid, T.pipes * 128, smem, s>>>(c->P, T, R, L);
       MF_CUDA(cudaGetLastError());
     }
   }

@@ -60,6 +60,7 @@ static void free_ctx(mf_ctx* c) {
   cudaFree(c->d_tc);
   cudaFree(c->d_partial);
   cudaFree(c->d_fc);
+  cudaFree(c->d_util);
   cudaFree(c->d_scratch);
   cudaFree(c->d_pop[0]);
   cudaFree(c->d_pop[1]);
@@ -157,6 +158,7 @@ mf_status mf_create(const mf_problem* p, mf_ctx** out) {
   P.h2 = p->hidden2;
   P.d_in = p->d_local + 4;
   P.objective = p->objective;
+  c->base_objective = p->objective;
   P.out_act = p->out_act;
   P.vram_cap = p->vram_cap;
   P.soft_penalty = p->soft_penalty;
@@ -263,6 +265,49 @@ mf_status mf_destroy(mf_ctx* ctx) {
 mf_status mf_space_size(const mf_ctx* ctx, uint64_t* out) {
   if (!ctx || !out) return einval("NULL argument");
   *out = ctx->P.total;
+  return MF_OK;
+}
+
+mf_status mf_set_utility(mf_ctx* ctx, const mf_fc_params* p) {
+  g_last_error.clear();
+  if (!ctx) return einval("ctx is NULL");
+  DeviceGuard guard(ctx->device);
+  Params& P = ctx->P;
+  if (!p) {  // back to the problem's own objective
+    P.objective = ctx->base_objective;
+    ctx->params_version++;
+    return MF_OK;
+  }
+  if (!p->variant || !p->quality || !p->f_min || !p->f_max || !p->omega || !p->tau || !p->reload_cost ||
+      !p->prev_variant)
+    return einval("mf_fc_params: every array but obs is required");
+  const int N = P.n_models, sumK = ctx->sumK;
+  std::vector<float4> tab(sumK);
+  for (int r = 0; r < sumK; ++r) {
+    if (!(p->f_max[r] > p->f_min[r])) return einval("mf_fc_params: f_max must exceed f_min for every option");
+    if (p->variant[r] < 0) return einval("mf_fc_params: variants must be >= 0");
+    float v;
+    std::memcpy(&v, &p->variant[r], sizeof(float));
+    tab[r] = make_float4(p->f_min[r], p->f_max[r] - p->f_min[r], p->quality[r], v);
+  }
+  for (int i = 0; i < N; ++i)
+    if (p->prev_variant[i] < -1) return einval("mf_fc_params: prev_variant must be >= -1");
+  if (!std::isfinite(p->alpha) || !std::isfinite(p->beta) || !std::isfinite(p->delta))
+    return einval("mf_fc_params: alpha, beta and delta must be finite");
+  if (!ctx->d_util) MF_CUDA(cudaMalloc(&ctx->d_util, sizeof(float4) * (size_t)sumK));
+  MF_CUDA(cudaMemcpy(ctx->d_util, tab.data(), sizeof(float4) * (size_t)sumK, cudaMemcpyHostToDevice));
+  P.util = ctx->d_util;
+  for (int i = 0; i < N; ++i) {
+    P.u_omega[i] = p->omega[i];
+    P.u_tau[i] = p->tau[i];
+    P.u_cost[i] = p->reload_cost[i];
+    P.u_prev[i] = p->prev_variant[i];
+  }
+  P.u_alpha = p->alpha;
+  P.u_beta = p->beta;
+  P.u_delta = p->delta;
+  P.objective = MF_OBJ_UTILITY;
+  ctx->params_version++;
   return MF_OK;
 }
 

@@ -33,6 +33,11 @@ struct Params {
   const float* w32;                   // predictors, packed as given
   const float* wT;                    // predictors with W1, W2 transposed ([in][out])
   uint32_t* status;                   // device status word (bit 0: bad index/gene)
+  // Eq. 3 utility (objective MF_OBJ_UTILITY)
+  const float4* util;                 // [sumK] (f_min, f_max - f_min, Q, variant as int bits)
+  float u_omega[MF_MAX_MODELS], u_tau[MF_MAX_MODELS], u_cost[MF_MAX_MODELS];
+  int32_t u_prev[MF_MAX_MODELS];
+  float u_alpha, u_beta, u_delta;
 };
 
 // Tensor-core path: operand images and the per-CTA layout (filled by tc_prepare).
@@ -88,12 +93,36 @@ __device__ __forceinline__ float out_act(const Params& P, float v) {
 }
 
 // Objective and constraints of one candidate from per-model outputs.
+// Model i's term of the Eq. 3 utility from its predicted throughput fhat (after the
+// output activation) for option row `row`: per-variant normalisation, quality,
+// reload cost when the variant changes, quadratic margin below tau_i + delta.
+// *f: the normalised throughput (its floor is tau_i).
+__device__ __forceinline__ float util_term_of(const Params& P, float4 q, float omega, float tau, float cost,
+                                             int prev, float fhat, float* f) {
+  const float fn = (fhat - q.x) / q.y;
+  const int v = __float_as_int(q.w);
+  const float eta = (prev >= 0 && v != prev) ? 1.f : 0.f;
+  const float margin = tau + P.u_delta - fn;
+  *f = fn;
+  return omega * fn * q.z - P.u_alpha * eta * cost - P.u_beta * (margin > 0.f ? margin * margin : 0.f);
+}
+
+__device__ __forceinline__ float util_term(const Params& P, int i, int row, float fhat, float* f) {
+  return util_term_of(P, P.util[row], P.u_omega[i], P.u_tau[i], P.u_cost[i], P.u_prev[i], fhat, f);
+}
+
 struct Acc {
   float J, pen;
-  bool sla_ok;
+  bool sla_ok;    // latency ceilings (weighted throughput) or floors (utility)
   __device__ __forceinline__ void init() { J = 0.f; pen = 0.f; sla_ok = true; }
-  // thr, lat: predictor outputs after the output activation.
-  __device__ __forceinline__ void add(const Params& P, int i, float thr, float lat) {
+  // thr, lat: predictor outputs after the output activation; row: the option row.
+  __device__ __forceinline__ void add(const Params& P, int i, float thr, float lat, int row) {
+    if (P.objective == MF_OBJ_UTILITY) {
+      float f;
+      J += util_term(P, i, row, thr, &f);
+      sla_ok = sla_ok && (f >= P.u_tau[i]);
+      return;
+    }
     J = fmaf(P.w[i], thr, J);
     sla_ok = sla_ok && (lat <= P.sla[i]);
     float over = lat - P.sla[i];
@@ -102,8 +131,8 @@ struct Acc {
   // Returns feasibility; J becomes the final score (-inf when infeasible).
   __device__ __forceinline__ bool finish(const Params& P, float vram_sum) {
     bool feas = vram_sum <= P.vram_cap;
-    if (P.objective == MF_OBJ_WEIGHTED_THR) feas = feas && sla_ok;
-    else J = fmaf(-P.soft_penalty, pen, J);
+    if (P.objective == MF_OBJ_SOFT_LAT) J = fmaf(-P.soft_penalty, pen, J);
+    else feas = feas && sla_ok;
     if (J != J) feas = false;
     if (!feas) J = -INFINITY;
     return feas;
@@ -220,6 +249,8 @@ struct mf_ctx {
   // fixed-context mode: the per-option table of the last mf_fc_set
   void* d_fc = nullptr;           // see mf::FcLayout
   int fc_ready = 0;
+  float4* d_util = nullptr;       // [sumK] utility table of mf_set_utility
+  int32_t base_objective = 0;     // the problem's own objective
   size_t tc_bytes = 0;
   mf::TcArgs tc{};
   // growable scratch (search lists, merge buffers, shortlist)

@@ -25,7 +25,7 @@ _EXPORTS = ["mf_status_string", "mf_last_error", "mf_create", "mf_destroy", "mf_
             "mf_set_objective", "mf_score_batch", "mf_search_range", "mf_search_exhaustive",
             "mf_ga_generation", "mf_ga_init", "mf_ga_step", "mf_ga_run", "mf_check_device_status",
             "mf_get_stats", "mf_search_exhaustive_noalloc", "mf_fc_set", "mf_fc_table", "mf_fc_search",
-            "mf_vram_feasible"]
+            "mf_vram_feasible", "mf_set_utility"]
 
 
 class MFError(RuntimeError):
@@ -94,6 +94,7 @@ def _load() -> C.CDLL:
     lib.mf_fc_table.argtypes = [vp, vp, vp, vp, vp, vp]
     lib.mf_fc_search.argtypes = [vp, u64, u64, i32, u64, C.POINTER(_Result), vp]
     lib.mf_vram_feasible.argtypes = [vp, u64, u64, vp, u64, C.POINTER(u64), vp]
+    lib.mf_set_utility.argtypes = [vp, C.POINTER(_FcParams)]
     for name in _EXPORTS[2:]:
         getattr(lib, name).restype = st
     return lib
@@ -277,8 +278,8 @@ class Context:
         return float(fit.value), genome
 
     # -- fixed-context mode ---------------------------------------------------
-    def fc_set(self, fc: dict) -> None:
-        """Evaluate the local predictions under fc["obs"] and build the utility table."""
+    @staticmethod
+    def _fc_params(fc: dict):
         keep = {
             "obs": np.ascontiguousarray(fc["obs"], dtype=np.float32),
             "variant": np.ascontiguousarray(fc["variant"], dtype=np.int32),
@@ -293,7 +294,20 @@ class Context:
         p = _FcParams(*(keep[k].ctypes.data for k in ("obs", "variant", "quality", "f_min", "f_max", "omega",
                                                        "tau", "reload_cost", "prev_variant")),
                       float(fc["alpha"]), float(fc["beta"]), float(fc["delta"]))
+        return p, keep
+
+    def fc_set(self, fc: dict) -> None:
+        """Evaluate the local predictions under fc["obs"] and build the utility table."""
+        p, keep = self._fc_params(fc)
         _check(_lib.mf_fc_set(self._h, C.byref(p), _stream(self.device)), "mf_fc_set")
+
+    def set_utility(self, fc: dict | None) -> None:
+        """Score with the Eq. 3 utility on the coupled aggregate (None: the problem's objective)."""
+        if fc is None:
+            _check(_lib.mf_set_utility(self._h, None), "mf_set_utility")
+            return
+        p, keep = self._fc_params(dict(fc, obs=np.zeros(4, np.float32)))
+        _check(_lib.mf_set_utility(self._h, C.byref(p)), "mf_set_utility")
 
     def fc_table(self):
         """(fhat, f, u, ok) of every option row, as numpy arrays."""
