@@ -670,3 +670,107 @@ void orc_util_exhaustive(const orc_problem *p, const orc_fc *fc, uint64_t lo, ui
   }
   *count = total_count;
 }
+
+/* ---------------------------------------------------------------------------
+ * The paper's GA (Sec. IV-C) on the fixed-context landscape (Sec. III-B holds s_t
+ * fixed during the GA search).
+ * ------------------------------------------------------------------------- */
+enum { GA_CROSS_DO = 6, GA_REPAIR = 7 };
+
+/* J of a genome from the per-option terms (the sum over models of Eq. 3's terms,
+ * -inf when a floor fails or the VRAM bound of Eq. 4 is exceeded). */
+static double fc_fitness(const orc_problem *p, const double *u, const int32_t *ok, const int32_t *o) {
+  double J = 0.0, vram = 0.0;
+  int32_t good = 1;
+  for (int32_t i = 0; i < p->n_models; ++i) {
+    const int64_t r = option_offset(p, i) + o[i];
+    J += u[r];
+    good = good && ok[r];
+    vram += (double)p->demand[3 * r + 1];
+  }
+  return (good && vram <= (double)p->vram_cap && !isnan(J)) ? J : -INFINITY;
+}
+
+/* Repair: replace an infeasible genome by a uniformly drawn feasible one (rejection,
+ * at most floor(256 / N) attempts, draws (gen, slot, GA_REPAIR, a * N + i)). */
+static double fc_repair(const orc_problem *p, const double *u, const int32_t *ok, uint64_t seed, uint32_t gen,
+                        uint32_t slot, int32_t *o, double J) {
+  const int32_t n = p->n_models;
+  const int32_t attempts = 256 / n;
+  int32_t cand[64];
+  for (int32_t a = 0; a < attempts && J == -INFINITY; ++a) {
+    for (int32_t i = 0; i < n; ++i)
+      cand[i] = unif_int(orc_rng(seed, gen, slot, GA_REPAIR, (uint32_t)(a * n + i)), (uint32_t)p->n_options[i]);
+    const double Jc = fc_fitness(p, u, ok, cand);
+    if (Jc != -INFINITY) {
+      memcpy(o, cand, sizeof(int32_t) * (size_t)n);
+      J = Jc;
+    }
+  }
+  return J;
+}
+
+double orc_fc_ga_run(const orc_problem *p, const orc_fc *fc, const orc_fc_ga_params *g, uint64_t seed,
+                     int32_t *best_genome) {
+  const int32_t n = p->n_models;
+  int64_t rows = 0;
+  for (int32_t i = 0; i < n; ++i) rows += p->n_options[i];
+  double *fhat = (double *)malloc(sizeof(double) * (size_t)rows);
+  double *f = (double *)malloc(sizeof(double) * (size_t)rows);
+  double *u = (double *)malloc(sizeof(double) * (size_t)rows);
+  int32_t *ok = (int32_t *)malloc(sizeof(int32_t) * (size_t)rows);
+  orc_fc_local(p, fc, fhat, f, ok, u);
+  int32_t *pop = (int32_t *)malloc(sizeof(int32_t) * (size_t)g->pop * n);
+  int32_t *next = (int32_t *)malloc(sizeof(int32_t) * (size_t)g->pop * n);
+  double *fit = (double *)malloc(sizeof(double) * (size_t)g->pop);
+  double *nfit = (double *)malloc(sizeof(double) * (size_t)g->pop);
+  const uint32_t mut_thr = (uint32_t)floor(g->mutation_p * 16777216.0 + 0.5);
+  const uint32_t cross_thr = (uint32_t)floor(g->crossover_p * 16777216.0 + 0.5);
+  /* initial population: uniform over Lambda, repaired */
+  for (int32_t c = 0; c < g->pop; ++c) {
+    int32_t *o = pop + (int64_t)c * n;
+    for (int32_t i = 0; i < n; ++i)
+      o[i] = unif_int(orc_rng(seed, 0, (uint32_t)c, GA_INIT, (uint32_t)i), (uint32_t)p->n_options[i]);
+    fit[c] = fc_fitness(p, u, ok, o);
+    if (g->repair) fit[c] = fc_repair(p, u, ok, seed, 0, (uint32_t)c, o, fit[c]);
+  }
+  for (int32_t gen = 0; gen + 1 < g->gens; ++gen) {
+    const uint32_t G = (uint32_t)gen + 1u;
+    int32_t first = 0;
+    if (g->elitism) {
+      int32_t e = 0;
+      for (int32_t c = 1; c < g->pop; ++c)
+        if (fit[c] > fit[e]) e = c;
+      memcpy(next, pop + (int64_t)e * n, sizeof(int32_t) * (size_t)n);
+      nfit[0] = fit[e];
+      first = 1;
+    }
+    for (int32_t c = first; c < g->pop; ++c) {
+      const orc_ga_params tg = {g->pop, g->gens, g->tournament, g->mutation_p, g->elitism};
+      const int32_t a = tournament(&tg, fit, seed, G, (uint32_t)c, GA_TOUR_A);
+      const int32_t b = tournament(&tg, fit, seed, G, (uint32_t)c, GA_TOUR_B);
+      /* crossover with probability crossover_p, else a copy of the first parent */
+      const int32_t cross = (uint32_t)(orc_rng(seed, G, (uint32_t)c, GA_CROSS_DO, 0) >> 40) < cross_thr;
+      int32_t *o = next + (int64_t)c * n;
+      for (int32_t i = 0; i < n; ++i) {
+        const uint64_t rc = orc_rng(seed, G, (uint32_t)c, GA_CROSS, (uint32_t)i);
+        int32_t gene = (cross && (rc >> 63)) ? pop[(int64_t)b * n + i] : pop[(int64_t)a * n + i];
+        const uint64_t rm = orc_rng(seed, G, (uint32_t)c, GA_MUT, (uint32_t)i);
+        if ((uint32_t)(rm >> 40) < mut_thr)
+          gene = unif_int(orc_rng(seed, G, (uint32_t)c, GA_MUTVAL, (uint32_t)i), (uint32_t)p->n_options[i]);
+        o[i] = gene;
+      }
+      nfit[c] = fc_fitness(p, u, ok, o);
+      if (g->repair) nfit[c] = fc_repair(p, u, ok, seed, G, (uint32_t)c, o, nfit[c]);
+    }
+    memcpy(pop, next, sizeof(int32_t) * (size_t)g->pop * n);
+    memcpy(fit, nfit, sizeof(double) * (size_t)g->pop);
+  }
+  int32_t e = 0;
+  for (int32_t c = 1; c < g->pop; ++c)
+    if (fit[c] > fit[e]) e = c;
+  memcpy(best_genome, pop + (int64_t)e * n, sizeof(int32_t) * (size_t)n);
+  const double J = fit[e];
+  free(fhat); free(f); free(u); free(ok); free(pop); free(next); free(fit); free(nfit);
+  return J;
+}

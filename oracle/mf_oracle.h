@@ -23,6 +23,9 @@
  *                                     reload term = alpha c, quadratic margin term,
  *                                     linear case as one matrix product)
  *   orc_vram_feasible                 pinned (two-pointer count, brute-force list)
+ *   orc_fc_ga_run                     pinned by properties (near-optimal decisions on the
+ *                                     paper-scale space, repair reaches feasibility,
+ *                                     seeding); the trajectory itself is parity unpinned
  *   orc_util_*                        pinned (hand example, equal to the fixed-context
  *                                     utility when the aggregate is unused, reduces to
  *                                     the weighted-throughput objective)
@@ -148,6 +151,28 @@ void orc_util_score_list(const orc_problem *p, const orc_fc *fc, const uint64_t 
                          double *score, int32_t *feasible, double *pred, double *agg, int32_t nthreads);
 void orc_util_exhaustive(const orc_problem *p, const orc_fc *fc, uint64_t lo, uint64_t hi, int32_t k,
                          uint64_t *topk_idx, double *topk_score, uint64_t *count, int32_t nthreads);
+
+/* The paper's GA (Sec. IV-C) on the fixed-context landscape: tournament selection,
+ * uniform crossover applied with probability crossover_p (else the first parent is
+ * copied), per-gene mutation, elitism, and repair of an infeasible individual
+ * (J = -inf) by a randomly sampled feasible one.  Reading: the sample is drawn by
+ * rejection from the uniform distribution over Lambda, at most floor(256 / N)
+ * attempts (the individual stays infeasible if none succeeds); the initial
+ * population is uniform over Lambda and repaired the same way. */
+typedef struct {
+  int32_t pop;
+  int32_t gens;
+  int32_t tournament;
+  double crossover_p;
+  double mutation_p;
+  int32_t elitism;          /* 0 or 1 */
+  int32_t repair;           /* 0 or 1 */
+} orc_fc_ga_params;
+
+/* Returns the best fitness of the last population (lowest slot among equals) and
+ * its genome in best_genome[N]. */
+double orc_fc_ga_run(const orc_problem *p, const orc_fc *fc, const orc_fc_ga_params *g, uint64_t seed,
+                     int32_t *best_genome);
 
 /* The VRAM-feasible joint configurations in [lo, hi) (Lambda with the
  * VRAM-infeasible configurations removed), ascending; writes at most cap of

@@ -57,6 +57,12 @@ class _FC(C.Structure):
                 ("alpha", C.c_float), ("beta", C.c_float), ("delta", C.c_float)]
 
 
+class _FcGAParams(C.Structure):
+    _fields_ = [("pop", C.c_int32), ("gens", C.c_int32), ("tournament", C.c_int32),
+                ("crossover_p", C.c_double), ("mutation_p", C.c_double), ("elitism", C.c_int32),
+                ("repair", C.c_int32)]
+
+
 class _GAParams(C.Structure):
     _fields_ = [("pop", C.c_int32), ("gens", C.c_int32), ("tournament", C.c_int32),
                 ("mutation_p", C.c_double), ("elitism", C.c_int32)]
@@ -96,6 +102,8 @@ def _load():
             lib.orc_util_score_list.restype = None
             lib.orc_util_exhaustive.argtypes = [P, F, u64, u64, i32, vp, vp, vp, i32]
             lib.orc_util_exhaustive.restype = None
+            lib.orc_fc_ga_run.argtypes = [P, F, C.POINTER(_FcGAParams), u64, vp]
+            lib.orc_fc_ga_run.restype = dbl
             _lib = lib
     return _lib
 
@@ -281,6 +289,16 @@ class Oracle:
         self.lib.orc_util_exhaustive(C.byref(self.p), C.byref(f_), int(lo), hi, int(k), _ptr(ti), _ptr(ts),
                                      _ptr(cnt), self.nthreads)
         return ti, ts, int(cnt[0])
+
+    def fc_ga_run(self, fc: dict, params: dict, seed: int):
+        """The paper's GA on the fixed-context landscape: (best J, genome)."""
+        f_ = self._fc(fc)
+        g = _FcGAParams(int(params["pop"]), int(params["gens"]), int(params["tournament"]),
+                        float(params["crossover_p"]), float(params["mutation_p"]), int(params["elitism"]),
+                        int(params["repair"]))
+        best = np.zeros(self.n, dtype=np.int32)
+        J = self.lib.orc_fc_ga_run(C.byref(self.p), C.byref(f_), C.byref(g), int(seed), _ptr(best))
+        return float(J), best
 
     def vram_feasible(self, lo: int = 0, hi: int | None = None, cap: int | None = None):
         """(count, ascending list of the first min(count, cap) VRAM-feasible indices)."""

@@ -265,6 +265,11 @@ def fc_scenario(prob: dict, seed: int) -> dict:
                 alpha=1.0 / 60.0, beta=5.0, delta=0.05)
 
 
+# The paper's GA at N = 5 (Sec. IV-C): 100 candidates, crossover probability 0.7,
+# mutation probability 0.1, tournament of 3, elitism, 30 generations; infeasible
+# offspring are repaired.
+PAPER_GA_PARAMS = dict(pop=100, gens=30, tournament=3, crossover_p=0.7, mutation_p=0.1, elitism=1, repair=1)
+
 GA_SCENARIO_SEEDS = tuple(range(100, 108))
 GA_RUN_SEEDS = tuple(range(1000, 1050))
 

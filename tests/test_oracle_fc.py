@@ -218,3 +218,54 @@ def test_util_reduces_to_weighted_throughput(oracle_mod):
     b, fb = r.score_list(idx)
     assert np.array_equal(fa, fb) and fa.all()
     np.testing.assert_allclose(a, b, rtol=1e-12, atol=1e-15)
+
+
+# ---------------------------------------------------------------------------
+# The paper's GA on the fixed-context landscape
+# ---------------------------------------------------------------------------
+
+def test_paper_ga_finds_the_optimum_of_the_paper_space(oracle_mod):
+    """Pop 100, 30 generations (Sec. IV-C) on the 78,732-configuration space: the
+    decision is within 0.5 % of the exhaustive optimum for every seed tried (the paper
+    reports 0.10 % average, 0.38 % worst gap)."""
+    prob = W.paper_scale()
+    o = oracle_mod.Oracle(prob)
+    for sc in (3, 6):
+        fc = W.fc_scenario(prob, sc)
+        _, ts, _ = o.fc_exhaustive(fc, 1)
+        for seed in (1000, 1001, 1002):
+            J, g = o.fc_ga_run(fc, W.PAPER_GA_PARAMS, seed)
+            assert o.fc_score_digits(fc, g) == (J, True)
+            assert J >= ts[0] - 0.005 * abs(ts[0])
+
+
+def test_paper_ga_repair_reaches_a_feasible_decision(oracle_mod):
+    """High floors leave a small feasible set: without repair the random population
+    holds no feasible individual and the decision is infeasible; with repair
+    (rejection sampling) it is feasible."""
+    prob = W.paper_scale()
+    o = oracle_mod.Oracle(prob)
+    fc = W.fc_scenario(prob, 3)
+    _, f, _, _ = o.fc_local(fc)
+    off = np.concatenate([[0], np.cumsum(prob["n_options"])])
+    # each model's floor just below its second-best normalised throughput: 2 feasible options per model
+    tau = np.array([np.sort(f[off[i]:off[i + 1]])[-2] - 1e-6 for i in range(5)], np.float32)
+    hard = dict(fc, tau=tau)
+    _, _, cnt = o.fc_exhaustive(hard, 1)
+    assert 0 < cnt <= 32
+    g0 = dict(W.PAPER_GA_PARAMS, repair=0, mutation_p=0.0, gens=2)
+    J0, _ = o.fc_ga_run(hard, g0, 5)
+    assert J0 == -np.inf
+    J1, g1 = o.fc_ga_run(hard, dict(W.PAPER_GA_PARAMS, gens=2), 5)
+    assert np.isfinite(J1) and o.fc_score_digits(hard, g1)[1]
+
+
+def test_paper_ga_is_deterministic_and_seeded(oracle_mod):
+    prob = W.paper_scale()
+    o = oracle_mod.Oracle(prob)
+    fc = W.fc_scenario(prob, 6)
+    g = dict(W.PAPER_GA_PARAMS, gens=3)
+    a = o.fc_ga_run(fc, g, 11)
+    assert a[0] == o.fc_ga_run(fc, g, 11)[0] and np.array_equal(a[1], o.fc_ga_run(fc, g, 11)[1])
+    outs = {tuple(o.fc_ga_run(fc, g, s)[1]) for s in range(11, 19)}
+    assert len(outs) > 1  # three generations do not always reach the same configuration
