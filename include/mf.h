@@ -254,6 +254,29 @@ mf_status mf_fc_table(mf_ctx *ctx, float *d_fhat, float *d_f, float *d_u, uint8_
 mf_status mf_fc_search(mf_ctx *ctx, uint64_t lo, uint64_t hi, int32_t k, uint64_t chunk, mf_result *out,
                        void *stream);
 
+/* The paper's GA (Sec. IV-C) on the fixed-context landscape of the last mf_fc_set:
+ * tournament selection, uniform crossover applied with probability crossover_p (else
+ * a copy of the first parent), per-gene mutation, elitism, and repair of an
+ * infeasible individual (J = -inf) by a feasible one drawn by rejection from the
+ * uniform distribution over Lambda (at most floor(256 / N) attempts; the initial
+ * uniform population is repaired the same way).  Fitness is the table sum of
+ * mf_fc_search (fp32).  Random draws: the counter-based generator of mf_ga_step
+ * plus purposes 6 (crossover coin) and 7 (repair, j = attempt * N + gene).
+ * Result (host): the fittest individual of the last population, lowest slot among
+ * equals.  Synchronous.  One CTA: pop <= 1024. */
+typedef struct {
+  int32_t pop;                 /* 2..1024 */
+  int32_t gens;                /* >= 1 fitness evaluations */
+  int32_t tournament;          /* 1..256 */
+  double crossover_p;          /* [0, 1]; paper 0.7 */
+  double mutation_p;           /* [0, 1]; paper 0.1 */
+  int32_t elitism;             /* 0 or 1 */
+  int32_t repair;              /* 0 or 1 */
+} mf_fc_ga_params;
+
+mf_status mf_fc_ga_run(mf_ctx *ctx, const mf_fc_ga_params *g, uint64_t seed, int32_t *best_genome,
+                       float *best_fitness, void *stream);
+
 /* Lambda without its VRAM-infeasible configurations (Eq. 4 applied when Lambda is
  * built): writes the ascending indices of [lo, hi) whose summed VRAM <= vram_cap to
  * d_out (device, capacity cap; indices beyond cap are counted, not written) and

@@ -380,6 +380,119 @@ static void radix_digits(const Params& P, uint64_t v, uint32_t* step) {
   }
 }
 
+// ---------------------------------------------------------------------------
+// The paper's GA (Sec. IV-C) on the fixed-context landscape, one CTA: thread c keeps
+// individual c; fitness is the table sum of fc mode.  Operators and draws follow the
+// GA of k_ga.cu with two more: crossover applied with probability crossover_p (draw
+// kGaCrossDo, else the first parent is copied) and repair of an infeasible individual
+// by rejection sampling from the uniform distribution over Lambda (draws kGaRepair,
+// j = a * N + i, at most 256 / N attempts).
+// ---------------------------------------------------------------------------
+struct FcGaArgs {
+  const float2* tab;
+  int pop, gens, tournament, elitism, repair;
+  uint32_t mut_thr, cross_thr;     // 24-bit thresholds
+  uint64_t seed;
+  int32_t* out_genome;
+  float* out_fit;
+};
+
+__device__ __forceinline__ float fc_fit(const Params& P, const float2* tab, const uint8_t* g) {
+  float J = 0.f, V = 0.f;
+  for (int i = 0; i < P.n_models; ++i) {
+    const float2 e = tab[pick(P.off, i) + g[i]];
+    J += e.x;
+    V += e.y;
+  }
+  return (V <= P.vram_cap && J > -INFINITY) ? J : -INFINITY;
+}
+
+__global__ void __launch_bounds__(1024)
+k_fc_ga(const Params P, const FcGaArgs A) {
+  extern __shared__ __align__(16) unsigned char sm[];
+  __shared__ float sval[32];
+  __shared__ int sidx[32];
+  const int N = P.n_models, pop = A.pop;
+  const int sumK = pick(P.off, N - 1) + pick(P.K, N - 1);
+  float2* tab = reinterpret_cast<float2*>(sm);
+  float* fit0 = reinterpret_cast<float*>(tab + sumK);
+  float* fit1 = fit0 + pop;
+  uint8_t* g0 = reinterpret_cast<uint8_t*>(fit1 + pop);
+  uint8_t* g1 = g0 + (size_t)pop * N;
+  const int c = threadIdx.x;
+  for (int e = c; e < sumK; e += blockDim.x) tab[e] = A.tab[e];
+  __syncthreads();
+  const uint64_t sd = A.seed;
+  const int attempts = 256 / N;
+  auto repair = [&](uint32_t G, uint8_t* g, float J) -> float {
+    uint8_t cand[MF_MAX_MODELS];
+    for (int a = 0; a < attempts && J == -INFINITY; ++a) {
+      for (int i = 0; i < N; ++i)
+        cand[i] = (uint8_t)ga_unif(ga_rng(sd, G, (uint32_t)c, kGaRepair, (uint32_t)(a * N + i)), (uint32_t)pick(P.K, i));
+      const float Jc = fc_fit(P, tab, cand);
+      if (Jc != -INFINITY) {
+        for (int i = 0; i < N; ++i) g[i] = cand[i];
+        J = Jc;
+      }
+    }
+    return J;
+  };
+  if (c < pop) {  // initial population: uniform over Lambda, repaired
+    uint8_t* g = g0 + (size_t)c * N;
+    for (int i = 0; i < N; ++i) g[i] = (uint8_t)ga_unif(ga_rng(sd, 0, (uint32_t)c, kGaInit, (uint32_t)i), (uint32_t)pick(P.K, i));
+    float J = fc_fit(P, tab, g);
+    if (A.repair) J = repair(0u, g, J);
+    fit0[c] = J;
+  }
+  __syncthreads();
+  uint8_t* gc = g0;
+  uint8_t* gn = g1;
+  float* fc_ = fit0;
+  float* fn = fit1;
+  for (int gen = 0; gen + 1 < A.gens; ++gen) {
+    const uint32_t G = (uint32_t)gen + 1u;
+    int first = 0;
+    if (A.elitism) {  // slot 0 keeps the fittest (lowest slot among equals)
+      const int e = block_argmax(fc_, pop, sval, sidx);
+      if (c < N) gn[c] = gc[(size_t)e * N + c];
+      if (c == 0) fn[0] = fc_[e];
+      first = 1;
+    }
+    if (c >= first && c < pop) {
+      int win[2];
+      for (int w = 0; w < 2; ++w) {
+        int best = -1;
+        float bf = 0.f;
+        for (int t = 0; t < A.tournament; ++t) {
+          const int s2 = ga_unif(ga_rng(sd, G, (uint32_t)c, w ? kGaTourB : kGaTourA, (uint32_t)t), (uint32_t)pop);
+          const float f = fc_[s2];
+          if (best < 0 || f > bf || (f == bf && s2 < best)) { best = s2; bf = f; }
+        }
+        win[w] = best;
+      }
+      const bool cross = (uint32_t)(ga_rng(sd, G, (uint32_t)c, kGaCrossDo, 0u) >> 40) < A.cross_thr;
+      uint8_t* g = gn + (size_t)c * N;
+      for (int i = 0; i < N; ++i) {
+        const uint64_t rc = ga_rng(sd, G, (uint32_t)c, kGaCross, (uint32_t)i);
+        uint8_t gene = (cross && (rc >> 63)) ? gc[(size_t)win[1] * N + i] : gc[(size_t)win[0] * N + i];
+        const uint64_t rm = ga_rng(sd, G, (uint32_t)c, kGaMut, (uint32_t)i);
+        if ((uint32_t)(rm >> 40) < A.mut_thr)
+          gene = (uint8_t)ga_unif(ga_rng(sd, G, (uint32_t)c, kGaMutVal, (uint32_t)i), (uint32_t)pick(P.K, i));
+        g[i] = gene;
+      }
+      float J = fc_fit(P, tab, g);
+      if (A.repair) J = repair(G, g, J);
+      fn[c] = J;
+    }
+    __syncthreads();
+    uint8_t* tg = gc; gc = gn; gn = tg;
+    float* tf = fc_; fc_ = fn; fn = tf;
+  }
+  const int e = block_argmax(fc_, pop, sval, sidx);
+  if (c < N) A.out_genome[c] = gc[(size_t)e * N + c];
+  if (c == 0) *A.out_fit = fc_[e];
+}
+
 int fc_grid(const mf_ctx* c) { return c->num_sms; }
 
 mf_status fc_search_chunk(mf_ctx* c, const RangeArgs& a, cudaStream_t s) {
@@ -512,5 +625,52 @@ mf_status mf_vram_feasible(mf_ctx* ctx, uint64_t lo, uint64_t hi, uint64_t* d_ou
   MF_CUDA(cudaMemcpyAsync(h, counts + grid, sizeof(unsigned long long), cudaMemcpyDeviceToHost, s));
   MF_CUDA(cudaStreamSynchronize(s));
   *count = *h;
+  return MF_OK;
+}
+
+mf_status mf_fc_ga_run(mf_ctx* ctx, const mf_fc_ga_params* g, uint64_t seed, int32_t* best_genome,
+                       float* best_fitness, void* stream) {
+  set_error("");
+  if (!ctx || !g || !best_genome || !best_fitness) return fc_einval("NULL argument");
+  if (!ctx->fc_ready) return fc_einval("mf_fc_set has not been called on this context");
+  if (g->pop < 2 || g->pop > 1024) return fc_einval("pop must be in 2..1024");
+  if (g->gens < 1) return fc_einval("gens must be >= 1");
+  if (g->tournament < 1 || g->tournament > 256) return fc_einval("tournament must be in 1..256");
+  if (!(g->crossover_p >= 0.0 && g->crossover_p <= 1.0) || !(g->mutation_p >= 0.0 && g->mutation_p <= 1.0))
+    return fc_einval("crossover_p and mutation_p must be in [0, 1]");
+  if ((g->elitism != 0 && g->elitism != 1) || (g->repair != 0 && g->repair != 1))
+    return fc_einval("elitism and repair must be 0 or 1");
+  DeviceGuard guard(ctx->device);
+  cudaStream_t s = (cudaStream_t)stream;
+  const int N = ctx->P.n_models;
+  FcLayout L;
+  fc_bytes(ctx->sumK, N, &L, (char*)ctx->d_fc);
+  // result: genome (16 ints) then the fitness
+  mf_status st = ensure_scratch(ctx, sizeof(int32_t) * 17);
+  if (st != MF_OK) return st;
+  st = ensure_host_stage(ctx, sizeof(int32_t) * 17);
+  if (st != MF_OK) return st;
+  FcGaArgs A{};
+  A.tab = L.tab;
+  A.pop = g->pop;
+  A.gens = g->gens;
+  A.tournament = g->tournament;
+  A.elitism = g->elitism;
+  A.repair = g->repair;
+  A.mut_thr = (uint32_t)std::floor(g->mutation_p * 16777216.0 + 0.5);
+  A.cross_thr = (uint32_t)std::floor(g->crossover_p * 16777216.0 + 0.5);
+  A.seed = seed;
+  A.out_genome = (int32_t*)ctx->d_scratch;
+  A.out_fit = (float*)((int32_t*)ctx->d_scratch + 16);
+  const size_t smem = sizeof(float2) * ctx->sumK + sizeof(float) * 2 * g->pop + (size_t)2 * g->pop * N;
+  const int threads = (g->pop + 31) / 32 * 32;
+  MF_CUDA(cudaFuncSetAttribute(k_fc_ga, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+  k_fc_ga<<<1, threads, smem, s>>>(ctx->P, A);
+  MF_CUDA(cudaGetLastError());
+  int32_t* h = (int32_t*)ctx->h_stage;
+  MF_CUDA(cudaMemcpyAsync(h, ctx->d_scratch, sizeof(int32_t) * 17, cudaMemcpyDeviceToHost, s));
+  MF_CUDA(cudaStreamSynchronize(s));
+  std::memcpy(best_genome, h, sizeof(int32_t) * N);
+  std::memcpy(best_fitness, h + 16, sizeof(float));
   return MF_OK;
 }

@@ -22,38 +22,6 @@ __global__ void k_ga_init(GaArgs g, const uint64_t* __restrict__ seed_ptr, uint6
   pop[e] = ga_unif(ga_rng(sd, 0, (uint32_t)c, kGaInit, (uint32_t)i), (uint32_t)g.K[i]);
 }
 
-// Index of the fittest individual, lowest slot among equals (block-wide).
-__device__ int block_argmax(const float* __restrict__ fit, int P, float* sval, int* sidx) {
-  float best = -INFINITY;
-  int bi = 0x7fffffff;
-  for (int c = threadIdx.x; c < P; c += blockDim.x) {
-    const float f = fit[c];
-    if (bi == 0x7fffffff || f > best || (f == best && c < bi)) { best = f; bi = c; }
-  }
-  for (int o = 16; o > 0; o >>= 1) {
-    const float ob = __shfl_xor_sync(0xffffffffu, best, o);
-    const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-    if (oi != 0x7fffffff && (bi == 0x7fffffff || ob > best || (ob == best && oi < bi))) { best = ob; bi = oi; }
-  }
-  const int w = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
-  if ((threadIdx.x & 31) == 0) { sval[w] = best; sidx[w] = bi; }
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    float b = sval[0];
-    int x = sidx[0];
-    for (int j = 1; j < nw; ++j)
-      if (sidx[j] != 0x7fffffff && (x == 0x7fffffff || sval[j] > b || (sval[j] == b && sidx[j] < x))) {
-        b = sval[j]; x = sidx[j];
-      }
-    sval[0] = b;
-    sidx[0] = x;
-  }
-  __syncthreads();
-  const int r = sidx[0];
-  __syncthreads();
-  return r;
-}
-
 __device__ __forceinline__ int tournament(const GaArgs& g, const float* __restrict__ fit, uint64_t seed,
                                           uint32_t gen, uint32_t child, uint32_t purpose) {
   int best = -1;

@@ -159,6 +159,39 @@ __device__ __forceinline__ T pick(const T (&a)[MF_MAX_MODELS], int i) {
   return v;
 }
 
+// Index of the fittest individual of fit[0, n), lowest slot among equals (block-wide;
+// every thread of the block calls it; sval/sidx: 32 entries of shared memory).
+__device__ __forceinline__ int block_argmax(const float* __restrict__ fit, int n, float* sval, int* sidx) {
+  float best = -INFINITY;
+  int bi = 0x7fffffff;
+  for (int c = threadIdx.x; c < n; c += blockDim.x) {
+    const float f = fit[c];
+    if (bi == 0x7fffffff || f > best || (f == best && c < bi)) { best = f; bi = c; }
+  }
+  for (int o = 16; o > 0; o >>= 1) {
+    const float ob = __shfl_xor_sync(0xffffffffu, best, o);
+    const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+    if (oi != 0x7fffffff && (bi == 0x7fffffff || ob > best || (ob == best && oi < bi))) { best = ob; bi = oi; }
+  }
+  const int w = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+  if ((threadIdx.x & 31) == 0) { sval[w] = best; sidx[w] = bi; }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float b = sval[0];
+    int x = sidx[0];
+    for (int j = 1; j < nw; ++j)
+      if (sidx[j] != 0x7fffffff && (x == 0x7fffffff || sval[j] > b || (sval[j] == b && sidx[j] < x))) {
+        b = sval[j]; x = sidx[j];
+      }
+    sval[0] = b;
+    sidx[0] = x;
+  }
+  __syncthreads();
+  const int r = sidx[0];
+  __syncthreads();
+  return r;
+}
+
 // SplitMix64 output number ctr of the sequence whose state starts at seed
 // (Steele, Lea and Flood, OOPSLA 2014).
 __device__ __forceinline__ uint64_t splitmix64(uint64_t seed, uint64_t ctr) {
@@ -179,7 +212,8 @@ __device__ __forceinline__ int ga_unif(uint64_t r, uint32_t k) {
   return (int)(((r >> 32) * (uint64_t)k) >> 32);
 }
 
-enum { kGaInit = 0, kGaTourA = 1, kGaTourB = 2, kGaCross = 3, kGaMut = 4, kGaMutVal = 5 };
+enum { kGaInit = 0, kGaTourA = 1, kGaTourB = 2, kGaCross = 3, kGaMut = 4, kGaMutVal = 5, kGaCrossDo = 6,
+       kGaRepair = 7 };
 
 // ---------------------------------------------------------------------------
 // Per-CTA running top-k in shared memory (sorted by the total order), fed by

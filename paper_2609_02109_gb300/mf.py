@@ -25,7 +25,7 @@ _EXPORTS = ["mf_status_string", "mf_last_error", "mf_create", "mf_destroy", "mf_
             "mf_set_objective", "mf_score_batch", "mf_search_range", "mf_search_exhaustive",
             "mf_ga_generation", "mf_ga_init", "mf_ga_step", "mf_ga_run", "mf_check_device_status",
             "mf_get_stats", "mf_search_exhaustive_noalloc", "mf_fc_set", "mf_fc_table", "mf_fc_search",
-            "mf_vram_feasible", "mf_set_utility"]
+            "mf_vram_feasible", "mf_set_utility", "mf_fc_ga_run"]
 
 
 class MFError(RuntimeError):
@@ -69,6 +69,12 @@ class _FcParams(C.Structure):
                 ("alpha", C.c_float), ("beta", C.c_float), ("delta", C.c_float)]
 
 
+class _FcGAParams(C.Structure):
+    _fields_ = [("pop", C.c_int32), ("gens", C.c_int32), ("tournament", C.c_int32),
+                ("crossover_p", C.c_double), ("mutation_p", C.c_double), ("elitism", C.c_int32),
+                ("repair", C.c_int32)]
+
+
 def _load() -> C.CDLL:
     if not os.path.exists(LIB_PATH):
         raise ImportError(f"{LIB_PATH} is missing: build it with paper_2609_02109_gb300.build.build()")
@@ -95,6 +101,7 @@ def _load() -> C.CDLL:
     lib.mf_fc_search.argtypes = [vp, u64, u64, i32, u64, C.POINTER(_Result), vp]
     lib.mf_vram_feasible.argtypes = [vp, u64, u64, vp, u64, C.POINTER(u64), vp]
     lib.mf_set_utility.argtypes = [vp, C.POINTER(_FcParams)]
+    lib.mf_fc_ga_run.argtypes = [vp, C.POINTER(_FcGAParams), u64, vp, vp, vp]
     for name in _EXPORTS[2:]:
         getattr(lib, name).restype = st
     return lib
@@ -329,6 +336,17 @@ class Context:
                "mf_fc_search")
         return dict(best_idx=int(r.best_idx), best_score=float(r.best_score), count=int(r.feasible_count),
                     topk_idx=ti, topk_score=ts)
+
+    def fc_ga_run(self, params: dict, seed: int):
+        """The paper's GA on the fixed-context landscape: (best J, genome)."""
+        g = _FcGAParams(int(params["pop"]), int(params["gens"]), int(params["tournament"]),
+                        float(params["crossover_p"]), float(params["mutation_p"]), int(params["elitism"]),
+                        int(params["repair"]))
+        genome = np.zeros(self.n_models, dtype=np.int32)
+        fit = C.c_float()
+        _check(_lib.mf_fc_ga_run(self._h, C.byref(g), int(seed), genome.ctypes.data, C.byref(fit),
+                                 _stream(self.device)), "mf_fc_ga_run")
+        return float(fit.value), genome
 
     def vram_feasible(self, lo: int = 0, hi: int | None = None, cap: int | None = None):
         """(count, device tensor of the first min(count, cap) VRAM-feasible indices)."""

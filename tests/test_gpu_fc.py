@@ -149,3 +149,63 @@ def test_fc_errors(mf):
         with pytest.raises(mf.MFError) as e:
             ctx.fc_set(bad)
         assert e.value.status == mf.MF_EINVAL and "f_max" in str(e.value)
+
+
+# ---------------------------------------------------------------------------
+# The paper's GA on the fixed-context landscape
+# ---------------------------------------------------------------------------
+
+def _integer_fc(prob, seed):
+    """Utility inputs that keep every term an integer on an integer landscape:
+    f = fhat (f_min 0, f_max 1), Q and omega small integers, alpha = 1 with integer
+    reload costs, beta = 0; floors integers."""
+    fc = W.fc_scenario(prob, seed)
+    rows = int(prob["n_options"].sum())
+    n = int(prob["n_options"].size)
+    rs = np.random.default_rng(seed)
+    return dict(fc, f_min=np.zeros(rows, np.float32), f_max=np.ones(rows, np.float32),
+                quality=rs.integers(1, 3, rows).astype(np.float32), omega=rs.integers(1, 3, n).astype(np.float32),
+                reload_cost=rs.integers(1, 20, n).astype(np.float32), alpha=1.0, beta=0.0, delta=0.0,
+                tau=rs.integers(-150, 0, n).astype(np.float32))
+
+
+@pytest.mark.parametrize("opts,params", [
+    ([12, 9, 9, 9, 9], dict(W.PAPER_GA_PARAMS)),
+    ([12, 9, 9, 9, 9], dict(W.PAPER_GA_PARAMS, elitism=0, gens=12)),
+    ([16] * 4, dict(W.PAPER_GA_PARAMS, pop=1024, gens=20, tournament=4, crossover_p=1.0, mutation_p=0.05)),
+    ([5] * 8, dict(W.PAPER_GA_PARAMS, pop=37, repair=0)),
+    ([200], dict(W.PAPER_GA_PARAMS, pop=2, gens=1)),
+])
+def test_paper_ga_reproduces_the_oracle_exactly(mf, oracle_mod, opts, params):
+    """On an integer landscape every fitness is an exact integer, so the GPU run
+    must equal the oracle's run: same decision, same fitness."""
+    prob = W.integer_landscape(opts, 5, 5.0 * len(opts) + 5.0)
+    fc = _integer_fc(prob, 7)
+    o = oracle_mod.Oracle(prob)
+    _, _, cnt = o.fc_exhaustive(fc, 1)
+    assert 0 < cnt < o.space_size()
+    with mf.Context(prob) as ctx:
+        ctx.fc_set(fc)
+        for seed in (1000, 1001, 2 ** 40 + 9):
+            J, g = ctx.fc_ga_run(params, seed)
+            Jo, go = o.fc_ga_run(fc, params, seed)
+            assert list(g) == list(go) and J == Jo, (seed, g, go, J, Jo)
+
+
+def test_paper_ga_decisions_on_the_paper_landscape(mf, oracle_mod):
+    """The synthetic N = 5 landscape: every decision's oracle score equals its reported
+    fitness and is within 0.5 % of the exhaustive optimum."""
+    prob = W.paper_scale()
+    o = oracle_mod.Oracle(prob)
+    with mf.Context(prob) as ctx:
+        for sc in W.GA_SCENARIO_SEEDS[:4]:
+            fc = W.fc_scenario(prob, sc)
+            _, ts, cnt = o.fc_exhaustive(fc, 1)
+            if cnt == 0:
+                continue
+            ctx.fc_set(fc)
+            for seed in (1000, 1001):
+                J, g = ctx.fc_ga_run(W.PAPER_GA_PARAMS, seed)
+                Jo, feas = o.fc_score_digits(fc, g)
+                assert feas and abs(J - Jo) <= 1e-5 * max(1.0, abs(Jo))
+                assert Jo >= ts[0] - 0.005 * abs(ts[0])
