@@ -177,6 +177,17 @@ struct TcList {
   float* pred;
 };
 
+struct NamedSync128 {
+  int id;
+  __device__ void operator()() const { named_bar(id, 128); }
+};
+
+// The pipeline's top-k merge, out of line: it runs rarely and its registers stay off
+// the hot loop.
+__device__ __noinline__ void tc_topk_merge(const CtaTopK& tk, int row, int barid) {
+  topk_merge(tk, row, 128, NamedSync128{barid});
+}
+
 struct PipeWait {
   volatile int* abort;
   uint32_t* status;
@@ -210,9 +221,9 @@ __device__ __forceinline__ void mma_steps(int steps, uint32_t d_tmem, uint32_t a
 
 // KW: 32-bit words of an A1 row (8 or 16); AWO: word where the aggregate starts, or
 // -1 to take it from T at run time.  S1, S2, S3: K-steps of the three layers (0 = run time).
-// MP: the models run in several passes (T.m0..T.m1 and a partial record per candidate);
+// N3: columns of the layer-3 accumulator (16, or 0 = run time).  MP: the models run in several passes (T.m0..T.m1 and a partial record per candidate);
 // otherwise all N models in one launch.  UT: the Eq. 3 utility objective.
-template <int MODE, int KW, int AWO, int S1, int S2, int S3, bool MP, bool UT>
+template <int MODE, int KW, int AWO, int S1, int S2, int S3, int N3, bool MP, bool UT>
 __global__ void __launch_bounds__(kTcMaxPipes * 128, 1)
 k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   extern __shared__ __align__(1024) unsigned char smem[];
@@ -221,7 +232,8 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   __shared__ float s_b3[MF_MAX_MODELS][2];
   const int tid = threadIdx.x;
   // compile-time K-step counts must be the layout's (else no MMA may run)
-  if ((S1 > 0 && S1 != T.k1 / 16) || (S2 > 0 && S2 != T.h1 / 16 + 1) || (S3 > 0 && S3 != T.hl / 16)) {
+  if ((S1 > 0 && S1 != T.k1 / 16) || (S2 > 0 && S2 != T.h1 / 16 + 1) || (S3 > 0 && S3 != T.hl / 16) ||
+      (N3 > 0 && N3 != T.n3)) {
     if (tid == 0) atomicOr(P.status, kStatusBadInput);
     return;
   }
@@ -278,10 +290,10 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   }
   for (int e = tid; e < sumK; e += blockDim.x) dem_s[e] = P.dem[e];
 
-  // per-pipeline running top-k (range mode)
-  CtaTopK tk{};
+  // per-pipeline running top-k (range mode), its pointers rebuilt where they are used
   const int kcap = R.k;
-  if (MODE == kTcRange) {
+  auto topk = [&]() {
+    CtaTopK tk;
     unsigned char* q = smem + T.sm_topk +
                        (size_t)pipe * ((sizeof(uint64_t) + sizeof(float)) * (2 * (size_t)kcap + 128) + 16);
     tk.li = reinterpret_cast<uint64_t*>(q); q += sizeof(uint64_t) * kcap;
@@ -292,6 +304,10 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     tk.qs = reinterpret_cast<float*>(q); q += sizeof(float) * 128;
     tk.qn = reinterpret_cast<int*>(q);
     tk.k = kcap;
+    return tk;
+  };
+  if (MODE == kTcRange) {
+    const CtaTopK tk = topk();
     const size_t gl = ((size_t)blockIdx.x * npipes + pipe) * kcap;
     for (int e = row; e < kcap; e += 128) {
       tk.ls[e] = R.first ? -INFINITY : R.lists_s[gl + e];
@@ -330,6 +346,7 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   float thr_s = -INFINITY;
   uint64_t thr_i = kEmptyIdx;
   if (MODE == kTcRange) {
+    const CtaTopK tk = topk();
     thr_s = tk.ls[kcap - 1];
     thr_i = tk.li[kcap - 1];
   }
@@ -475,8 +492,11 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     await_mma();
 
     // ---- final epilogue: per-model outputs, constraints, objective ----
-    uint32_t d3[32];
-    if (T.n3 == 16) {
+    uint32_t d3[N3 == 16 ? 16 : 32];
+    if constexpr (N3 == 16) {
+      tmem_ld_x16(tD3 + lane_off, d3);
+      tmem_wait_ld();
+    } else if (T.n3 == 16) {
       uint32_t r16[16];
       tmem_ld_x16(tD3 + lane_off, r16);
       tmem_wait_ld();
@@ -494,7 +514,9 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
       if (i >= m1) break;
       if (i < m0) continue;
       const float thr = out_act(P, __uint_as_float(d3[i]) + s_b3[i][0]);
-      const float lat = out_act(P, __uint_as_float(half3 == 8 ? d3[(8 + i) & 31] : d3[(16 + i) & 31]) + s_b3[i][1]);
+      const float lat = out_act(P, __uint_as_float(N3 == 16 ? d3[(8 + i) & 15]
+                                                 : half3 == 8 ? d3[(8 + i) & 31] : d3[(16 + i) & 31]) +
+                                   s_b3[i][1]);
       if (MODE == kTcList && valid && L.pred) {
         L.pred[(t * N + i) * 2 + 0] = thr;
         L.pred[(t * N + i) * 2 + 1] = lat;
@@ -544,13 +566,14 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     } else {
       my_count += feas ? 1u : 0u;
       const bool push = cand && precedes(J, idx, thr_s, thr_i);
+      const CtaTopK tk = topk();
       if (push) {
         const int pos = atomicAdd(tk.qn, 1);
         tk.qs[pos] = J;
         tk.qi[pos] = idx;
       }
       if (named_bar_or(barid, 128, push)) {
-        topk_merge(tk, row, 128, [barid] __device__() { named_bar(barid, 128); });
+        tc_topk_merge(tk, row, barid);
         thr_s = tk.ls[kcap - 1];
         thr_i = tk.li[kcap - 1];
       }
@@ -558,6 +581,7 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   }
 
   if (MODE == kTcRange && (!MP || T.pass_last)) {
+    const CtaTopK tk = topk();
     const size_t gl = ((size_t)blockIdx.x * npipes + pipe) * kcap;
     for (int e = row; e < kcap; e += 128) {
       R.lists_s[gl + e] = tk.ls[e];
@@ -633,15 +657,17 @@ constexpr size_t kPassImageBudget = 160 * 1024;      // bf16 weights staged per 
 
 using TcFn = void (*)(const Params, const TcArgs, const RangeArgs, const TcList);
 
-// Instantiations: the two benchmark shapes (d_L 8, 64-64 and d_L 16, 128-128) with all
-// counts fixed at compile time, and a run-time fallback per A1 row width.
+// Instantiations: the two benchmark shapes (d_L 8, 64-64 and d_L 16, 128-128, up to 8
+// models) with all counts fixed at compile time, and a run-time fallback per A1 row width.
 template <int MODE, bool MP, bool UT>
 TcFn tc_kernel_mode(const TcArgs& T) {
   // S1 = k1 / 16, S2 = h1 / 16 + 1 (the b2 step), S3 = hl / 16
-  if (T.kw == 8 && T.dle == 8 && T.h1 == 64 && T.h2 == 64) return k_score_tc<MODE, 8, 4, 1, 5, 4, MP, UT>;
-  if (T.kw == 16 && T.dle == 16 && T.h1 == 128 && T.h2 == 128) return k_score_tc<MODE, 16, 8, 2, 9, 8, MP, UT>;
-  if (T.kw == 8) return k_score_tc<MODE, 8, -1, 0, 0, 0, MP, UT>;
-  return k_score_tc<MODE, 16, -1, 0, 0, 0, MP, UT>;
+  if (T.kw == 8 && T.dle == 8 && T.h1 == 64 && T.h2 == 64 && T.n3 == 16)
+    return k_score_tc<MODE, 8, 4, 1, 5, 4, 16, MP, UT>;
+  if (T.kw == 16 && T.dle == 16 && T.h1 == 128 && T.h2 == 128 && T.n3 == 16)
+    return k_score_tc<MODE, 16, 8, 2, 9, 8, 16, MP, UT>;
+  if (T.kw == 8) return k_score_tc<MODE, 8, -1, 0, 0, 0, 0, MP, UT>;
+  return k_score_tc<MODE, 16, -1, 0, 0, 0, 0, MP, UT>;
 }
 
 template <bool UT>
