@@ -336,7 +336,7 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   const int m0 = MP ? T.m0 : 0, m1 = MP ? T.m1 : N;  // this pass's models
   const float vcap = P.vram_cap;
 
-  {  // constant ones block: word 0 = (1, 1) feeds the bias hi/lo rows of B2 and B3
+  {  // constant ones block: word 0 = (1, 1) feeds the bias hi/lo rows of B2
     uint32_t v[8] = {0x3F803F80u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
     tmem_st_x8(tOnes + lane_off, v);
     tmem_wait_st();
