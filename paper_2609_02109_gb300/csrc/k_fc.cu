@@ -381,12 +381,13 @@ static void radix_digits(const Params& P, uint64_t v, uint32_t* step) {
 }
 
 // ---------------------------------------------------------------------------
-// The paper's GA (Sec. IV-C) on the fixed-context landscape, one CTA: thread c keeps
+// The paper's GA (Sec. IV-C) on the fixed-context landscape, one CTA: thread c breeds
 // individual c; fitness is the table sum of fc mode.  Operators and draws follow the
 // GA of k_ga.cu with two more: crossover applied with probability crossover_p (draw
 // kGaCrossDo, else the first parent is copied) and repair of an infeasible individual
 // by rejection sampling from the uniform distribution over Lambda (draws kGaRepair,
-// j = a * N + i, at most 256 / N attempts).
+// j = a * N + i, at most 256 / N attempts, the first feasible one kept).  A warp's
+// repairs share its lanes (see repair_warp).
 // ---------------------------------------------------------------------------
 struct FcGaArgs {
   const float2* tab;
@@ -424,26 +425,70 @@ k_fc_ga(const Params P, const FcGaArgs A) {
   __syncthreads();
   const uint64_t sd = A.seed;
   const int attempts = 256 / N;
-  auto repair = [&](uint32_t G, uint8_t* g, float J) -> float {
-    uint8_t cand[MF_MAX_MODELS];
-    for (int a = 0; a < attempts && J == -INFINITY; ++a) {
-      for (int i = 0; i < N; ++i)
-        cand[i] = (uint8_t)ga_unif(ga_rng(sd, G, (uint32_t)c, kGaRepair, (uint32_t)(a * N + i)), (uint32_t)pick(P.K, i));
-      const float Jc = fc_fit(P, tab, cand);
-      if (Jc != -INFINITY) {
-        for (int i = 0; i < N; ++i) g[i] = cand[i];
-        J = Jc;
+  // Repair of the warp's infeasible children (need): the m of them (rounded up to a
+  // power of two) each get a group of 32 / m lanes, which tries the child's attempts
+  // 32 / m at a time; the lowest feasible attempt of a group's first successful round is
+  // the sequential search's result.  The winning lane writes the child's genes and
+  // fitness over the unrepaired ones already in shared memory.  With 32 pending
+  // children this is the sequential search on every lane.
+  const int lane = c & 31;
+  auto repair_warp = [&](uint32_t G, bool need, uint8_t* genes, float* fit) {
+    __syncwarp();
+    const unsigned pend = __ballot_sync(0xffffffffu, need);
+    if (!pend) return;
+    const int cnt = __popc(pend);
+    int m = 1;
+    while (m < cnt) m <<= 1;
+    const int gs = 32 / m, grp = lane / gs, lig = lane % gs;
+    int child = -1;
+    if (grp < cnt) {
+      unsigned x = pend;
+      for (int q = 0; q < grp; ++q) x &= x - 1;
+      child = (c & ~31) + __ffs(x) - 1;
+    }
+    const unsigned gmask = gs == 32 ? 0xffffffffu : ((1u << gs) - 1u) << (grp * gs);
+    bool done = child < 0;
+    for (int a0 = 0; a0 < attempts; a0 += gs) {
+      if (!__any_sync(0xffffffffu, !done)) break;
+      const int a = a0 + lig;
+      float Jc = -INFINITY;
+      uint8_t cand[MF_MAX_MODELS];
+      if (!done && a < attempts) {  // fc_fit's sums, with the draws kept in registers
+        float Js = 0.f, Vs = 0.f;
+#pragma unroll
+        for (int i = 0; i < MF_MAX_MODELS; ++i) {
+          if (i < N) {
+            cand[i] = (uint8_t)ga_unif(ga_rng(sd, G, (uint32_t)child, kGaRepair, (uint32_t)(a * N + i)),
+                                       (uint32_t)pick(P.K, i));
+            const float2 e = tab[pick(P.off, i) + cand[i]];
+            Js += e.x;
+            Vs += e.y;
+          }
+        }
+        Jc = (Vs <= P.vram_cap && Js > -INFINITY) ? Js : -INFINITY;
+      }
+      const unsigned ok = __ballot_sync(0xffffffffu, Jc != -INFINITY) & gmask;
+      if (!done && ok) {
+        if (lane == __ffs(ok) - 1) {
+#pragma unroll
+          for (int i = 0; i < MF_MAX_MODELS; ++i)
+            if (i < N) genes[(size_t)child * N + i] = cand[i];
+          fit[child] = Jc;
+        }
+        done = true;
       }
     }
-    return J;
+    __syncwarp();
   };
+  bool need = false;
   if (c < pop) {  // initial population: uniform over Lambda, repaired
     uint8_t* g = g0 + (size_t)c * N;
     for (int i = 0; i < N; ++i) g[i] = (uint8_t)ga_unif(ga_rng(sd, 0, (uint32_t)c, kGaInit, (uint32_t)i), (uint32_t)pick(P.K, i));
-    float J = fc_fit(P, tab, g);
-    if (A.repair) J = repair(0u, g, J);
+    const float J = fc_fit(P, tab, g);
     fit0[c] = J;
+    need = A.repair && J == -INFINITY;
   }
+  repair_warp(0u, need, g0, fit0);
   __syncthreads();
   uint8_t* gc = g0;
   uint8_t* gn = g1;
@@ -458,6 +503,7 @@ k_fc_ga(const Params P, const FcGaArgs A) {
       if (c == 0) fn[0] = fc_[e];
       first = 1;
     }
+    need = false;
     if (c >= first && c < pop) {
       int win[2];
       for (int w = 0; w < 2; ++w) {
@@ -480,10 +526,11 @@ k_fc_ga(const Params P, const FcGaArgs A) {
           gene = (uint8_t)ga_unif(ga_rng(sd, G, (uint32_t)c, kGaMutVal, (uint32_t)i), (uint32_t)pick(P.K, i));
         g[i] = gene;
       }
-      float J = fc_fit(P, tab, g);
-      if (A.repair) J = repair(G, g, J);
+      const float J = fc_fit(P, tab, g);
       fn[c] = J;
+      need = A.repair && J == -INFINITY;
     }
+    repair_warp(G, need, gn, fn);
     __syncthreads();
     uint8_t* tg = gc; gc = gn; gn = tg;
     float* tf = fc_; fc_ = fn; fn = tf;
