@@ -245,7 +245,9 @@ k_fc_scan(const Params P, const FcScan S, const RangeArgs R) {
       }
     }
     if (__syncthreads_or(any)) {  // block-uniform
-      topk_merge(tk, tid, blockDim.x, [] __device__() { __syncthreads(); });
+      // a queue that fills a whole run (the first runs of a search) is sorted first
+      if (*tk.qn > 256) topk_merge_sorted(tk, tid, blockDim.x, [] __device__() { __syncthreads(); });
+      else topk_merge(tk, tid, blockDim.x, [] __device__() { __syncthreads(); });
       thr_s = tk.ls[R.k - 1];
       thr_i = tk.li[R.k - 1];
     }

@@ -259,6 +259,64 @@ __device__ void topk_merge(const CtaTopK& t, int tid, int nthr, Sync sync) {
   sync();
 }
 
+// The same merge for a long queue (up to qcap entries, qcap a power of two): the queue
+// is first sorted best-first by a bitonic network over the next power of two (padding
+// entries are (-inf, empty), last in the order), so an entry's rank is its position in
+// the sorted queue plus the number of list entries ahead of it, found by binary search
+// (and a list entry's rank likewise).  O(q log^2 q) work instead of O(q k).
+template <class Sync>
+__device__ void topk_merge_sorted(const CtaTopK& t, int tid, int nthr, Sync sync) {
+  const int k = t.k;
+  const int q = *t.qn;
+  int n2 = 1;
+  while (n2 < q) n2 <<= 1;
+  for (int e = q + tid; e < n2; e += nthr) { t.qs[e] = -INFINITY; t.qi[e] = kEmptyIdx; }
+  for (int e = tid; e < k; e += nthr) { t.ns[e] = -INFINITY; t.ni[e] = kEmptyIdx; }
+  sync();
+  for (int size = 2; size <= n2; size <<= 1) {
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      for (int i = tid; i < (n2 >> 1); i += nthr) {
+        const int a = 2 * stride * (i / stride) + (i % stride), b = a + stride;
+        const float sa = t.qs[a], sb = t.qs[b];
+        const uint64_t ia = t.qi[a], ib = t.qi[b];
+        const bool best_first = (a & size) == 0;
+        if (best_first ? precedes(sb, ib, sa, ia) : precedes(sa, ia, sb, ib)) {
+          t.qs[a] = sb; t.qi[a] = ib;
+          t.qs[b] = sa; t.qi[b] = ia;
+        }
+      }
+      sync();
+    }
+  }
+  // queue entries: only the first k positions can rank below k
+  for (int p = tid; p < k && p < q; p += nthr) {
+    const float s = t.qs[p];
+    const uint64_t id = t.qi[p];
+    int lo = 0, hi = k;
+    while (lo < hi) {
+      const int mid = (lo + hi) >> 1;
+      if (precedes(t.ls[mid], t.li[mid], s, id)) lo = mid + 1; else hi = mid;
+    }
+    if (p + lo < k) { t.ns[p + lo] = s; t.ni[p + lo] = id; }
+  }
+  // list entries
+  for (int e = tid; e < k; e += nthr) {
+    const float s = t.ls[e];
+    const uint64_t id = t.li[e];
+    if (id == kEmptyIdx) continue;
+    int lo = 0, hi = q;
+    while (lo < hi) {
+      const int mid = (lo + hi) >> 1;
+      if (precedes(t.qs[mid], t.qi[mid], s, id)) lo = mid + 1; else hi = mid;
+    }
+    if (e + lo < k) { t.ns[e + lo] = s; t.ni[e + lo] = id; }
+  }
+  sync();
+  for (int e = tid; e < k; e += nthr) { t.ls[e] = t.ns[e]; t.li[e] = t.ni[e]; }
+  if (tid == 0) *t.qn = 0;
+  sync();
+}
+
 }  // namespace mf
 
 // ---------------------------------------------------------------------------
