@@ -139,23 +139,28 @@ k_fc_local(const Params P, const FcLayout L, const FcConst C) {
 }
 
 // ---------------------------------------------------------------------------
-// Table-lookup scan.  A step of the CTA covers 512 x kFcRun consecutive candidates:
-// thread t takes the run of kFcRun consecutive indices starting at step base + t *
-// kFcRun, so between them only the last model's option advances (the partial sum
+// Table-lookup scan.  A step of the CTA covers 512 x RUN consecutive candidates:
+// thread t takes the run of RUN consecutive indices starting at step base + t * RUN,
+// so between them only the last model's option advances (the partial sum
 // over the other models is reused until a carry).  J is summed in model order
 // either way.  Per-CTA running top-k as in the fp32 scorer, one merge check per
 // step with a queue of one entry per candidate of the step.
 // ---------------------------------------------------------------------------
 constexpr int kFcThreads = 512;
-constexpr int kFcRun = 8;
+// Runs of 16 halve the per-step barriers of long scans; runs of 8 keep the first step's
+// queue (every feasible candidate of the step, sorted before the merge) short.
+constexpr int kFcRunLong = 16, kFcRunShort = 8;
+constexpr uint64_t kFcLongScan = 1ull << 29;
 
 struct FcScan {
   const float2* tab;
-  uint32_t step[MF_MAX_MODELS];  // mixed-radix digits of the grid step (grid x threads x kFcRun)
+  uint32_t step[MF_MAX_MODELS];  // mixed-radix digits of the grid step (grid x threads x RUN)
 };
 
+template <int RUN>
 __global__ void __launch_bounds__(kFcThreads, 1)
 k_fc_scan(const Params P, const FcScan S, const RangeArgs R) {
+  constexpr int kFcRun = RUN;
   extern __shared__ __align__(16) unsigned char sm[];
   const int N = P.n_models;
   const int sumK = pick(P.off, N - 1) + pick(P.K, N - 1);
@@ -549,15 +554,18 @@ mf_status fc_search_chunk(mf_ctx* c, const RangeArgs& a, cudaStream_t s) {
   fc_bytes(c->sumK, c->P.n_models, &L, (char*)c->d_fc);
   FcScan S{};
   S.tab = L.tab;
-  radix_digits(c->P, (uint64_t)fc_grid(c) * kFcThreads * kFcRun, S.step);
+  const int run = a.len >= kFcLongScan ? kFcRunLong : kFcRunShort;
+  radix_digits(c->P, (uint64_t)fc_grid(c) * kFcThreads * run, S.step);
   const size_t smem = (((size_t)c->sumK * sizeof(float2) + 15) & ~(size_t)15) +
-                      (sizeof(uint64_t) + sizeof(float)) * (2 * (size_t)a.k + kFcThreads * kFcRun) + 16;
+                      (sizeof(uint64_t) + sizeof(float)) * (2 * (size_t)a.k + kFcThreads * run) + 16;
   if (smem > 227 * 1024) {
     set_error("fixed-context search: top-k lists do not fit shared memory; use a smaller k");
     return MF_EUNSUPPORTED;
   }
-  MF_CUDA(cudaFuncSetAttribute(k_fc_scan, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-  k_fc_scan<<<fc_grid(c), kFcThreads, smem, s>>>(c->P, S, a);
+  const void* fn = run == kFcRunLong ? (const void*)k_fc_scan<kFcRunLong> : (const void*)k_fc_scan<kFcRunShort>;
+  MF_CUDA(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+  if (run == kFcRunLong) k_fc_scan<kFcRunLong><<<fc_grid(c), kFcThreads, smem, s>>>(c->P, S, a);
+  else k_fc_scan<kFcRunShort><<<fc_grid(c), kFcThreads, smem, s>>>(c->P, S, a);
   MF_CUDA(cudaGetLastError());
   return MF_OK;
 }

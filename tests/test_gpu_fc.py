@@ -113,12 +113,13 @@ def test_vram_feasible_list_matches_oracle(mf, oracle_mod, name):
         assert gc2 == c2 and np.array_equal(gl2.cpu().numpy().astype(np.uint64), l2)
 
 
-@pytest.mark.parametrize("which,seed", [("large", 3), ("stress", 5)])
-def test_fc_full_size_separable_closed_form(mf, oracle_mod, which, seed):
+@pytest.mark.parametrize("which,seed,chunk", [("large", 3, 1 << 26), ("stress", 5, 1 << 30)])
+def test_fc_full_size_separable_closed_form(mf, oracle_mod, which, seed, chunk):
     """At full size (24^6 and 16^8 candidates) the VRAM cap of 180 GB never binds, so
     the feasible count is the product of the per-model floor-feasible option counts
     and the best configuration takes each model's best feasible option (from the
-    oracle's per-option table)."""
+    oracle's per-option table).  Chunks of 2^26 scan in runs of 8 candidates per
+    thread, chunks of 2^30 in runs of 16."""
     prob = W.large(precision="fp32") if which == "large" else W.stress(precision="fp32")
     fc = W.fc_scenario(prob, seed)
     o = oracle_mod.Oracle(prob)
@@ -133,7 +134,7 @@ def test_fc_full_size_separable_closed_form(mf, oracle_mod, which, seed):
         Jbest += float(np.max(ui))
     with mf.Context(prob) as ctx:
         ctx.fc_set(fc)
-        res = ctx.fc_search(16, chunk=1 << 26)
+        res = ctx.fc_search(16, chunk=chunk)
     assert res["count"] == count
     assert list(o.decode(res["best_idx"])) == best
     assert abs(res["best_score"] - Jbest) <= RTOL * max(1.0, float(np.abs(ru).sum()))
