@@ -282,8 +282,9 @@ k_score_f32(const Params P, const RangeArgs R, const ListArgs L) {
         tk.qi[pos] = idx;
       }
       // the barrier's OR is block-uniform, so every thread takes the same branch
-      if (__syncthreads_or(push)) {
-        topk_merge(tk, tid, blockDim.x, [] __device__() { __syncthreads(); });
+      if (__syncthreads_or(push)) {  // a long queue (early in a search) is sorted first
+        if (*tk.qn > 256) topk_merge_sorted(tk, tid, blockDim.x, [] __device__() { __syncthreads(); });
+        else topk_merge(tk, tid, blockDim.x, [] __device__() { __syncthreads(); });
         thr_s = tk.ls[R.k - 1];
         thr_i = tk.li[R.k - 1];
       }

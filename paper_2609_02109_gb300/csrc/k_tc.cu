@@ -478,10 +478,13 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
           issue_mma2(i);
           mma_commit(mbar);
         }
+        // layer 1 of model i has completed, so the next A1 goes in while layer 2 runs
+        if (i + 1 < m1) write_a1(i + 1);
         await_mma();
         epilogue(T.h2, tH2);  // layer 2 (bias through the ones block)
+      } else if (i + 1 < m1) {
+        write_a1(i + 1);
       }
-      if (i + 1 < m1) write_a1(i + 1);
       publish();
     }
     if (leader) {
