@@ -367,14 +367,14 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   auto issue_mma3 = [&](int i) { mma_steps<S3>(s3, tD3, tH2, desc_s[3 * i + 2], id3, i > m0 ? 1u : 0u); };
   // fp32 accumulators [0, width) -> ReLU -> bf16 pairs at dst
   auto epilogue = [&](int width, uint32_t dst) {
-    for (int c0 = 0; c0 < width; c0 += 32) {
-      uint32_t r[32];
-      tmem_ld_x32(tD + lane_off + c0, r);
+    for (int c0 = 0; c0 < width; c0 += 16) {
+      uint32_t r[16];
+      tmem_ld_x16(tD + lane_off + c0, r);
       tmem_wait_ld();
-      uint32_t h[16];
+      uint32_t h[8];
 #pragma unroll
-      for (int j = 0; j < 16; ++j) h[j] = relu_bf16x2(r[2 * j], r[2 * j + 1]);
-      tmem_st_x16(dst + lane_off + (c0 >> 1), h);
+      for (int j = 0; j < 8; ++j) h[j] = relu_bf16x2(r[2 * j], r[2 * j + 1]);
+      tmem_st_x8(dst + lane_off + (c0 >> 1), h);
     }
   };
 
