@@ -249,16 +249,19 @@ def fixed_context_throughput(mf, torch, device):
             ctx.fc_set(fc)
             set_ms = 1e3 * (time.perf_counter() - t0)
             ctx.fc_search(32, chunk=1 << 30)
-            e0 = torch.cuda.Event(enable_timing=True)
-            e1 = torch.cuda.Event(enable_timing=True)
-            torch.cuda.synchronize(device)
-            e0.record(stream)
-            res = ctx.fc_search(32, chunk=1 << 30)
-            e1.record(stream)
-            e1.synchronize()
-            st = ctx.stats()
-        ms = e0.elapsed_time(e1)
-        ops = 3 * N * n / (st["score_ms_last"] / 1e3)  # N table loads and 2N adds per candidate
+            times, scans = [], []
+            for _ in range(5):  # median of five searches
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                torch.cuda.synchronize(device)
+                e0.record(stream)
+                res = ctx.fc_search(32, chunk=1 << 30)
+                e1.record(stream)
+                e1.synchronize()
+                times.append(e0.elapsed_time(e1))
+                scans.append(ctx.stats()["score_ms_last"])
+        ms = float(np.median(times))
+        ops = 3 * N * n / (float(np.median(scans)) / 1e3)  # N table loads and 2N adds per candidate
         out[name] = {"candidates": n, "value": n / (ms / 1e3), "unit": UNIT, "ms": ms, "fc_set_ms": set_ms,
                      "count": res["count"],
                      "roofline": {"bound": "alu", "achieved": ops, "peak": issue, "unit": "lane-ops/s",

@@ -139,12 +139,11 @@ k_fc_local(const Params P, const FcLayout L, const FcConst C) {
 }
 
 // ---------------------------------------------------------------------------
-// Table-lookup scan.  A step of the CTA covers 512 x RUN consecutive candidates:
-// thread t takes the run of RUN consecutive indices starting at step base + t * RUN,
-// so between them only the last model's option advances (the partial sum
-// over the other models is reused until a carry).  J is summed in model order
-// either way.  Per-CTA running top-k as in the fp32 scorer, one merge check per
-// step with a queue of one entry per candidate of the step.
+// Table-lookup scan.  Each thread walks its own contiguous slice of the range, so from
+// one candidate to the next only the last model's option advances (the partial sum
+// over the other models is reused until a carry).  J is summed in model order either
+// way.  Per-CTA running top-k as in the fp32 scorer: every RUN candidates of each
+// thread, one merge check with a queue of one entry per candidate of the step.
 // ---------------------------------------------------------------------------
 constexpr int kFcThreads = 512;
 // Runs of 16 halve the per-step barriers of long scans; runs of 8 keep the first step's
@@ -154,7 +153,6 @@ constexpr uint64_t kFcLongScan = 1ull << 29;
 
 struct FcScan {
   const float2* tab;
-  uint32_t step[MF_MAX_MODELS];  // mixed-radix digits of the grid step (grid x threads x RUN)
 };
 
 template <int RUN>
@@ -177,21 +175,37 @@ k_fc_scan(const Params P, const FcScan S, const RangeArgs R) {
   tk.qs = reinterpret_cast<float*>(q); q += sizeof(float) * QCAP;
   tk.qn = reinterpret_cast<int*>(q);
   tk.k = R.k;
-  for (int e = tid; e < sumK; e += blockDim.x) tab[e] = S.tab[e];
+  // an option below its floor (utility -inf, or NaN) carries VRAM +inf here, so one
+  // compare against the cap decides feasibility
+  for (int e = tid; e < sumK; e += blockDim.x) {
+    float2 v = S.tab[e];
+    if (!(v.x > -INFINITY)) v.y = INFINITY;
+    tab[e] = v;
+  }
   const size_t gl = (size_t)blockIdx.x * R.k;
   for (int e = tid; e < R.k; e += blockDim.x) {
     tk.ls[e] = R.first ? -INFINITY : R.lists_s[gl + e];
     tk.li[e] = R.first ? kEmptyIdx : R.lists_i[gl + e];
   }
   if (tid == 0) *tk.qn = 0;
-  // digits of this thread's first run start
-  const uint64_t t0 = ((uint64_t)blockIdx.x * blockDim.x + tid) * kFcRun;
-  int start[MF_MAX_MODELS];
+  // Thread g of the grid scans the contiguous slice [g S, (g + 1) S) of the range, RUN
+  // candidates between two merge checks; its option rows, the prefix sum over models
+  // 0..N-2 and the last model's row carry from run to run.  S = ceil(len / threads); in
+  // long scans rounded up to a multiple of the last model's option count, so all lanes
+  // of a warp reach a carry at the same candidate (no divergence in the scan loop),
+  // while short scans keep slices short (a small first merge, spread over more CTAs).
+  const uint64_t nthreads = (uint64_t)gridDim.x * blockDim.x;
+  const uint64_t klast = (uint64_t)pick(P.K, N - 1);
+  const uint64_t slice0 = (R.len + nthreads - 1) / nthreads;
+  const uint64_t slice = slice0 >= 4 * klast ? (slice0 + klast - 1) / klast * klast : slice0;
+  const uint64_t s0 = ((uint64_t)blockIdx.x * blockDim.x + tid) * slice;
+  const uint64_t s1 = s0 + slice < R.len ? s0 + slice : R.len;
+  int row[MF_MAX_MODELS];
   {
-    const uint64_t idx0 = R.base + (t0 < R.len ? t0 : 0);
+    const uint64_t idx0 = R.base + (s0 < R.len ? s0 : 0);
 #pragma unroll
     for (int i = 0; i < MF_MAX_MODELS; ++i)
-      if (i < N) start[i] = P.off[i] + (int)((idx0 / P.stride[i]) % (uint64_t)P.K[i]);
+      if (i < N) row[i] = P.off[i] + (int)((idx0 / P.stride[i]) % (uint64_t)P.K[i]);
   }
   __syncthreads();
   float thr_s = tk.ls[R.k - 1];
@@ -201,36 +215,39 @@ k_fc_scan(const Params P, const FcScan S, const RangeArgs R) {
   const int off_last = pick(P.off, last);
   const int end_last = off_last + pick(P.K, last);
   unsigned int my_count = 0;
-  const uint64_t gstep = (uint64_t)gridDim.x * blockDim.x * kFcRun;
-  for (uint64_t base = (uint64_t)blockIdx.x * blockDim.x * kFcRun; base < R.len; base += gstep) {
-    // the run: rows from `start`, the prefix sum over models 0..N-2 until a carry
-    int row[MF_MAX_MODELS];
+  float pJ = 0.f, pV = 0.f;
 #pragma unroll
-    for (int i = 0; i < MF_MAX_MODELS; ++i) row[i] = start[i];
-    float pJ = 0.f, pV = 0.f;
-#pragma unroll
-    for (int i = 0; i < MF_MAX_MODELS; ++i)
-      if (i < last) { const float2 e = tab[row[i]]; pJ += e.x; pV += e.y; }
-    int rl = pick(row, last);
+  for (int i = 0; i < MF_MAX_MODELS; ++i)
+    if (i < last) { const float2 e = tab[row[i]]; pJ += e.x; pV += e.y; }
+  int rl = pick(row, last);
+  const uint64_t nruns = (slice + kFcRun - 1) / kFcRun;  // the same for every thread
+  for (uint64_t r = 0; r < nruns; ++r) {
     bool any = false;
-    const uint64_t t1 = base + (uint64_t)tid * kFcRun;
-#pragma unroll
-    for (int u = 0; u < kFcRun; ++u) {
-      const uint64_t t = t1 + u;
-      const float2 e = tab[rl];
-      const float J = pJ + e.x, V = pV + e.y;
-      // -inf below a floor; NaN compares false
-      const bool feas = t < R.len && V <= cap && J > -INFINITY;
-      const uint64_t idx = R.base + t;
-      my_count += feas ? 1u : 0u;
-      if (feas && precedes(J, idx, thr_s, thr_i)) {
-        const int pos = atomicAdd(tk.qn, 1);
-        tk.qs[pos] = J;
-        tk.qi[pos] = idx;
-        any = true;
+    const uint64_t t1 = s0 + r * kFcRun;
+    const int nv = t1 >= s1 ? 0 : (s1 - t1 >= (uint64_t)kFcRun ? kFcRun : (int)(s1 - t1));
+    // the run in segments between carries of the last model's option: a segment is a
+    // plain loop (one lookup, two adds, one compare per candidate); the carry into the
+    // prefix runs between segments
+    int u0 = 0;
+    while (u0 < nv) {
+      const int seg = min(nv - u0, end_last - rl);
+      for (int u = u0; u < u0 + seg; ++u, ++rl) {
+        const float2 e = tab[rl];
+        const float J = pJ + e.x, V = pV + e.y;
+        const bool feas = V <= cap;  // NaN compares false
+        my_count += feas ? 1u : 0u;
+        if (feas && J >= thr_s) {  // rare once the list is full; the index only then
+          const uint64_t idx = R.base + t1 + u;
+          if (precedes(J, idx, thr_s, thr_i)) {
+            const int pos = atomicAdd(tk.qn, 1);
+            tk.qs[pos] = J;
+            tk.qi[pos] = idx;
+            any = true;
+          }
+        }
       }
-      // next index: the last model's option, with a carry into the prefix
-      if (++rl == end_last) {
+      u0 += seg;
+      if (rl == end_last) {  // carry into the prefix
         rl = off_last;
         bool carry = true;
 #pragma unroll
@@ -256,18 +273,6 @@ k_fc_scan(const Params P, const FcScan S, const RangeArgs R) {
       thr_s = tk.ls[R.k - 1];
       thr_i = tk.li[R.k - 1];
     }
-    // advance the run start by the grid step, last model first
-    uint32_t carry = 0;
-#pragma unroll
-    for (int i = MF_MAX_MODELS - 1; i >= 0; --i)
-      if (i < N) {
-        const int off = P.off[i];
-        const uint32_t K = (uint32_t)P.K[i];
-        uint32_t d = (uint32_t)(start[i] - off) + S.step[i] + carry;
-        carry = d >= K;
-        if (carry) d -= K;
-        start[i] = off + (int)d;
-      }
   }
   for (int e = tid; e < R.k; e += blockDim.x) {
     R.lists_s[gl + e] = tk.ls[e];
@@ -555,7 +560,6 @@ mf_status fc_search_chunk(mf_ctx* c, const RangeArgs& a, cudaStream_t s) {
   FcScan S{};
   S.tab = L.tab;
   const int run = a.len >= kFcLongScan ? kFcRunLong : kFcRunShort;
-  radix_digits(c->P, (uint64_t)fc_grid(c) * kFcThreads * run, S.step);
   const size_t smem = (((size_t)c->sumK * sizeof(float2) + 15) & ~(size_t)15) +
                       (sizeof(uint64_t) + sizeof(float)) * (2 * (size_t)a.k + kFcThreads * run) + 16;
   if (smem > 227 * 1024) {
