@@ -44,7 +44,7 @@ L2_FLUSH_BYTES = 256 << 20
 # DRAM bytes (read + write) of one scoring launch from the ncu capture summarised in
 # profiles/k_score_tc_large_n6.md, valid only while the kernel's sources are the ones
 # that were captured (sha256 prefix of k_tc.cu + mf_internal.cuh)
-NCU_TRAFFIC = {"bf16": ("014c26756ca5ac7c", 2056448)}
+NCU_TRAFFIC = {"bf16": ("739c026bcbb59df6", 2116864)}
 
 
 def _traffic(prec):
