@@ -155,10 +155,10 @@ struct FcScan {
   const float2* tab;
 };
 
-template <int RUN>
+template <int RUN, int NMAX>
 __global__ void __launch_bounds__(kFcThreads, 1)
 k_fc_scan(const Params P, const FcScan S, const RangeArgs R) {
-  constexpr int kFcRun = RUN;
+  constexpr int kFcRun = RUN;  // NMAX: a bound on N for the unrolled per-model loops
   extern __shared__ __align__(16) unsigned char sm[];
   const int N = P.n_models;
   const int sumK = pick(P.off, N - 1) + pick(P.K, N - 1);
@@ -200,11 +200,11 @@ k_fc_scan(const Params P, const FcScan S, const RangeArgs R) {
   const uint64_t slice = slice0 >= 4 * klast ? (slice0 + klast - 1) / klast * klast : slice0;
   const uint64_t s0 = ((uint64_t)blockIdx.x * blockDim.x + tid) * slice;
   const uint64_t s1 = s0 + slice < R.len ? s0 + slice : R.len;
-  int row[MF_MAX_MODELS];
+  int row[NMAX];
   {
     const uint64_t idx0 = R.base + (s0 < R.len ? s0 : 0);
 #pragma unroll
-    for (int i = 0; i < MF_MAX_MODELS; ++i)
+    for (int i = 0; i < NMAX; ++i)
       if (i < N) row[i] = P.off[i] + (int)((idx0 / P.stride[i]) % (uint64_t)P.K[i]);
   }
   __syncthreads();
@@ -217,9 +217,12 @@ k_fc_scan(const Params P, const FcScan S, const RangeArgs R) {
   unsigned int my_count = 0;
   float pJ = 0.f, pV = 0.f;
 #pragma unroll
-  for (int i = 0; i < MF_MAX_MODELS; ++i)
+  for (int i = 0; i < NMAX; ++i)
     if (i < last) { const float2 e = tab[row[i]]; pJ += e.x; pV += e.y; }
-  int rl = pick(row, last);
+  int rl = row[0];
+#pragma unroll
+  for (int i = 1; i < NMAX; ++i)
+    if (i == last) rl = row[i];
   const uint64_t nruns = (slice + kFcRun - 1) / kFcRun;  // the same for every thread
   for (uint64_t r = 0; r < nruns; ++r) {
     bool any = false;
@@ -251,7 +254,7 @@ k_fc_scan(const Params P, const FcScan S, const RangeArgs R) {
         rl = off_last;
         bool carry = true;
 #pragma unroll
-        for (int i = MF_MAX_MODELS - 1; i >= 0; --i)
+        for (int i = NMAX - 1; i >= 0; --i)
           if (i < last && carry) {
             const int off = P.off[i];
             int d = row[i] - off + 1;
@@ -262,7 +265,7 @@ k_fc_scan(const Params P, const FcScan S, const RangeArgs R) {
         pJ = 0.f;
         pV = 0.f;
 #pragma unroll
-        for (int i = 0; i < MF_MAX_MODELS; ++i)
+        for (int i = 0; i < NMAX; ++i)
           if (i < last) { const float2 e2 = tab[row[i]]; pJ += e2.x; pV += e2.y; }
       }
     }
@@ -566,10 +569,12 @@ mf_status fc_search_chunk(mf_ctx* c, const RangeArgs& a, cudaStream_t s) {
     set_error("fixed-context search: top-k lists do not fit shared memory; use a smaller k");
     return MF_EUNSUPPORTED;
   }
-  const void* fn = run == kFcRunLong ? (const void*)k_fc_scan<kFcRunLong> : (const void*)k_fc_scan<kFcRunShort>;
+  using ScanFn = void (*)(const Params, const FcScan, const RangeArgs);
+  const bool small_n = c->P.n_models <= 8;
+  const ScanFn fn = run == kFcRunLong ? (small_n ? k_fc_scan<kFcRunLong, 8> : k_fc_scan<kFcRunLong, MF_MAX_MODELS>)
+                                      : (small_n ? k_fc_scan<kFcRunShort, 8> : k_fc_scan<kFcRunShort, MF_MAX_MODELS>);
   MF_CUDA(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-  if (run == kFcRunLong) k_fc_scan<kFcRunLong><<<fc_grid(c), kFcThreads, smem, s>>>(c->P, S, a);
-  else k_fc_scan<kFcRunShort><<<fc_grid(c), kFcThreads, smem, s>>>(c->P, S, a);
+  fn<<<fc_grid(c), kFcThreads, smem, s>>>(c->P, S, a);
   MF_CUDA(cudaGetLastError());
   return MF_OK;
 }

@@ -31,12 +31,15 @@ def _cases():
     tight = W.paper_scale()
     tight["vram_cap"] = 55.0  # binds: five options of 1-20 GB
     sig = W.random_small(21, n_models=4, max_options=8, h2=32, vram_cap=40.0, out_act="sigmoid")
+    sixteen = W.make_problem([2] * 16, 8, 32, 32, 33, 180.0)
     return {
         "hand": (W.hand_example(), _hand_fc()),
         "tiny": (W.tiny(), W.fc_scenario(W.tiny(), 4)),
         "paper": (W.paper_scale(), W.fc_scenario(W.paper_scale(), 3)),
         "paper_vram_binds": (tight, W.fc_scenario(tight, 6)),
         "sigmoid": (sig, W.fc_scenario(sig, 8)),
+        # sixteen models: the scan's loops over up to 16 models
+        "sixteen_models": (sixteen, W.fc_scenario(sixteen, 9)),
     }
 
 
