@@ -160,9 +160,17 @@ def cpu_baseline(prob, target_s=15.0):
         if dt >= 10.0 or n >= 24 ** 6:
             break
         n = int(min(n * max(2.0, target_s / max(dt, 1e-3)), 24 ** 6))
+    # one core, on a sample of about a fifth of that time
+    o1 = Oracle(prob, nthreads=1)
+    n1 = max(20000, n // (5 * max(cores, 1)))
+    t = time.perf_counter()
+    o1.exhaustive(K_TOP, lo=0, hi=n1)
+    dt1 = time.perf_counter() - t
     return {"value": n / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
             "sample": f"fp64 C oracle exhaustive search (top-32 + count) over indices [0, {n}) "
-                      f"of the same N=6 space, {dt:.1f} s"}
+                      f"of the same N=6 space, {dt:.1f} s",
+            "single_thread": {"value": n1 / dt1, "unit": UNIT, "cores": 1,
+                              "sample": f"indices [0, {n1}), {dt1:.1f} s"}}
 
 
 def run_reference(args):
