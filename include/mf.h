@@ -263,7 +263,8 @@ mf_status mf_fc_search(mf_ctx *ctx, uint64_t lo, uint64_t hi, int32_t k, uint64_
  * mf_fc_search (fp32).  Random draws: the counter-based generator of mf_ga_step
  * plus purposes 6 (crossover coin) and 7 (repair, j = attempt * N + gene).
  * Result (host): the fittest individual of the last population, lowest slot among
- * equals.  Synchronous.  One CTA: pop <= 1024. */
+ * equals; best_genome has N entries.  Synchronous.  One CTA: pop <= 1024.
+ * MF_EINVAL: NULL arguments, called before mf_fc_set, a parameter out of its range. */
 typedef struct {
   int32_t pop;                 /* 2..1024 */
   int32_t gens;                /* >= 1 fitness evaluations */
