@@ -149,6 +149,12 @@ __device__ __forceinline__ void tmem_ld_x32(uint32_t taddr, uint32_t (&r)[32]) {
                : "r"(taddr));
 }
 
+__device__ __forceinline__ void tmem_st_x4(uint32_t taddr, const uint32_t (&v)[4]) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x4.b32 [%0], {%1,%2,%3,%4};"
+               :: "r"(taddr), "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3])
+               : "memory");
+}
+
 __device__ __forceinline__ void tmem_st_x8(uint32_t taddr, const uint32_t (&v)[8]) {
   asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};"
                :: "r"(taddr), "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7])
@@ -188,44 +194,122 @@ __device__ __noinline__ void tc_topk_merge(const CtaTopK& tk, int row, int barid
   topk_merge(tk, row, 128, NamedSync128{barid});
 }
 
+// The rest of a bounded wait, out of line: on giving up it flags the status word and
+// every later wait returns at once, so the kernel still runs to its end.
+__device__ __noinline__ void mbar_wait_slow(uint64_t* bar, uint32_t parity, volatile int* abort, uint32_t* status) {
+  if (*abort) return;
+  uint32_t n = 0;
+  while (!mbar_try_wait(bar, parity)) {
+    if (++n == kWaitLimit) {
+      *abort = 1;
+      atomicOr(status, kStatusTimeout);
+      return;
+    }
+  }
+}
+
 struct PipeWait {
   volatile int* abort;
   uint32_t* status;
-  // Bounded wait for `parity` of `bar`; on giving up it flags the status word and
-  // every later wait returns at once, so the kernel still runs to its end.
+  // Bounded wait for `parity` of `bar` (the usual case is one suspended try).
   __device__ __forceinline__ void operator()(uint64_t* bar, uint32_t parity) const {
-    if (*abort) return;
-    uint32_t n = 0;
-    while (!mbar_try_wait(bar, parity)) {
-      if (++n == kWaitLimit) {
-        *abort = 1;
-        atomicOr(status, kStatusTimeout);
-        return;
-      }
-    }
+    if (!mbar_try_wait(bar, parity)) mbar_wait_slow(bar, parity, abort, status);
   }
 };
 
-// `steps` MMAs of K = 16 along one K extent; S > 0 unrolls a compile-time count (the
-// issuing thread's instruction stream is on the critical path of every round trip).
+// The predictor's output unit; the sigmoid out of line keeps the scorer's loop small.
+__device__ __noinline__ float tc_sigmoid(float v) { return 1.f / (1.f + expf(-v)); }
+__device__ __forceinline__ float tc_out(const Params& P, float v) {
+  return P.out_act == MF_ACT_SIGMOID ? tc_sigmoid(v) : v;
+}
+
+// MMA issue by a whole warp: every lane executes the instruction stream (so the
+// operands stay warp-uniform) and one elected lane issues.  The same lane is elected
+// for the MMAs and for the commit that tracks them.
+__device__ __forceinline__ void mma_ts_warp(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                                            uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p, e;\n setp.ne.b32 p, %4, 0;\n elect.sync _|e, 0xffffffff;\n"
+      " @e tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+__device__ __forceinline__ void mma_commit_warp(uint64_t* bar) {
+  asm volatile(
+      "{\n .reg .pred e;\n elect.sync _|e, 0xffffffff;\n"
+      " @e tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n}" ::"r"(smem_u32(bar))
+      : "memory");
+}
+
+// `steps` MMAs of K = 16 along one K extent; S > 0 unrolls a compile-time count.
 template <int S>
 __device__ __forceinline__ void mma_steps(int steps, uint32_t d_tmem, uint32_t a_tmem, uint64_t desc,
                                           uint32_t idesc, uint32_t acc0) {
   if constexpr (S > 0) {
 #pragma unroll
-    for (int s = 0; s < S; ++s) mma_ts(d_tmem, a_tmem + 8u * s, desc + 16u * s, idesc, s > 0 ? 1u : acc0);
+    for (int s = 0; s < S; ++s) mma_ts_warp(d_tmem, a_tmem + 8u * s, desc + 16u * s, idesc, s > 0 ? 1u : acc0);
   } else {
-    for (int s = 0; s < steps; ++s) mma_ts(d_tmem, a_tmem + 8u * s, desc + 16u * s, idesc, s > 0 ? 1u : acc0);
+    for (int s = 0; s < steps; ++s) mma_ts_warp(d_tmem, a_tmem + 8u * s, desc + 16u * s, idesc, s > 0 ? 1u : acc0);
+  }
+}
+
+// Hidden epilogue: fp32 accumulators [0, width) at `src` -> ReLU -> bf16 pairs at `dst`.
+// 64 columns are loaded before one wait.  `before_store` runs once, after the first
+// piece's loads and conversions and before its stores (round A waits there for the
+// previous model's layer 3, which reads the same tensor-memory columns).
+template <int W, class F>
+__device__ __forceinline__ void hidden_epilogue(int width, uint32_t src, uint32_t dst, F before_store) {
+  if constexpr (W > 0 && W % 64 == 0) {
+#pragma unroll 1
+    for (int c0 = 0; c0 < W; c0 += 64) {
+      uint32_t a[32], b[32];
+      tmem_ld_x32(src + c0, a);
+      tmem_ld_x32(src + c0 + 32, b);
+      tmem_wait_ld();
+      uint32_t h[16], g[16];
+#pragma unroll
+      for (int j = 0; j < 16; ++j) h[j] = relu_bf16x2(a[2 * j], a[2 * j + 1]);
+#pragma unroll
+      for (int j = 0; j < 16; ++j) g[j] = relu_bf16x2(b[2 * j], b[2 * j + 1]);
+      if (c0 == 0) before_store();
+      tmem_st_x16(dst + (c0 >> 1), h);
+      tmem_st_x16(dst + (c0 >> 1) + 16, g);
+    }
+  } else {
+    for (int c0 = 0; c0 < width; c0 += 32) {
+      uint32_t a[32];
+      tmem_ld_x32(src + c0, a);
+      tmem_wait_ld();
+      uint32_t h[16];
+#pragma unroll
+      for (int j = 0; j < 16; ++j) h[j] = relu_bf16x2(a[2 * j], a[2 * j + 1]);
+      if (c0 == 0) before_store();
+      tmem_st_x16(dst + (c0 >> 1), h);
+    }
   }
 }
 
 // KW: 32-bit words of an A1 row (8 or 16); AWO: word where the aggregate starts, or
 // -1 to take it from T at run time.  S1, S2, S3: K-steps of the three layers (0 = run time).
-// N3: columns of the layer-3 accumulator (16, or 0 = run time).  MP: the models run in several passes (T.m0..T.m1 and a partial record per candidate);
-// otherwise all N models in one launch.  UT: the Eq. 3 utility objective.
-template <int MODE, int KW, int AWO, int S1, int S2, int S3, int N3, bool MP, bool UT>
+// N3: columns of the layer-3 accumulator (16, or 0 = run time).  MP: the models run in
+// several passes (T.m0..T.m1 and a partial record per candidate); otherwise all N models
+// in one launch.  UT: the Eq. 3 utility objective.  NM: the number of models, when fixed at
+// compile time (0: run time); the per-model loop is then unrolled, so every per-model
+// offset, descriptor and branch is a constant.
+//
+// Per 128-row pipeline and model i the work is two rounds of MMAs:
+//   round A: layer 1 of model i (commit A) and layer 3 of model i - 1 (commit B; the
+//            last model's layer 3 of a tile rides in the next tile's first round A);
+//            epilogue: D1 -> H1, stored once layer 3 has finished reading H
+//   round B: layer 2 of model i (commit A); while it runs the next model's A1 is
+//            written (at the last model: the next tile's digits, aggregate and A1), and
+//            at the first model the previous tile's objective, constraints and top-k
+//            are finished from its layer-3 outputs; epilogue: D2 -> H2.
+template <int MODE, int KW, int AWO, int S1, int S2, int S3, int N3, bool MP, bool UT, int NM>
 __global__ void __launch_bounds__(kTcMaxPipes * 128, 1)
 k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
+  static_assert(AWO < 0 || AWO == 4 || AWO == 8, "partial A1 rows are written for these layouts only");
   extern __shared__ __align__(1024) unsigned char smem[];
   __shared__ uint32_t s_tmem;
   __shared__ int s_abort;
@@ -233,26 +317,29 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   const int tid = threadIdx.x;
   // compile-time K-step counts must be the layout's (else no MMA may run)
   if ((S1 > 0 && S1 != T.k1 / 16) || (S2 > 0 && S2 != T.h1 / 16 + 1) || (S3 > 0 && S3 != T.hl / 16) ||
-      (N3 > 0 && N3 != T.n3)) {
+      (N3 > 0 && N3 != T.n3) || (NM > 0 && (NM != P.n_models || MP))) {
     if (tid == 0) atomicOr(P.status, kStatusBadInput);
     return;
   }
-  const int warp = tid >> 5, lane = tid & 31;
+  // the warp index through a shuffle from lane 0, so the compiler knows it is warp-uniform
+  // and keeps everything derived from it (pipeline, tensor-memory addresses, issuer roles)
+  // in uniform registers with uniform branches
+  const int warp = __shfl_sync(0xffffffffu, tid >> 5, 0), lane = tid & 31;
   const int pipe = warp >> 2, wq = warp & 3;
   const int row = wq * 32 + lane;
-  const int N = P.n_models;
+  const int N = NM > 0 ? NM : P.n_models;
   const int npipes = T.pipes;
 
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + T.sm_bar);
   const uint4* xw_s = reinterpret_cast<const uint4*>(smem + T.sm_xw);
   float4* dem_s = reinterpret_cast<float4*>(smem + T.sm_dem);
-  uint64_t* desc_s = reinterpret_cast<uint64_t*>(smem + T.sm_desc);
-  // this thread's current option row of every model: rows[i * 128 + row]
-  uint16_t* rows = reinterpret_cast<uint16_t*>(smem + T.sm_rows) + (size_t)pipe * MF_MAX_MODELS * 128;
+  // this thread's digits (option index within the model) of every model, two tiles:
+  // digits[b * MF_MAX_MODELS * 128 + i * 128 + row]
+  uint8_t* digits = reinterpret_cast<uint8_t*>(smem + T.sm_rows) + (size_t)pipe * 2 * MF_MAX_MODELS * 128;
 
   if (tid == 0) {
     s_abort = 0;
-    for (int j = 0; j <= npipes; ++j) mbar_init(&bars[j], 1);
+    for (int j = 0; j < 1 + 2 * npipes; ++j) mbar_init(&bars[j], 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 0) {
@@ -271,12 +358,7 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
       bulk_g2s(smem + o, static_cast<const unsigned char*>(T.img) + T.img_lo + o, b, &bars[0]);
     }
   }
-  // UMMA descriptors of the pass's models' three B operands
   if (tid >= T.m0 && tid < T.m1) {
-    const uint32_t sb = smem_base - T.img_lo;
-    desc_s[3 * tid + 0] = smem_desc(sb + T.off_b1[tid], 128u, (uint32_t)(T.k1 / 8) * 128u);
-    desc_s[3 * tid + 1] = smem_desc(sb + T.off_b2[tid], 128u, (uint32_t)((T.h1 + 16) / 8) * 128u);
-    desc_s[3 * tid + 2] = smem_desc(sb + T.off_b3[tid], 128u, (uint32_t)(T.hl / 8) * 128u);
     const float* b3 = P.w32 + (size_t)tid * P.per_model + (size_t)T.h1 * P.d_in + T.h1 +
                       (T.h2 > 0 ? (size_t)T.h2 * T.h1 + T.h2 : 0) + 2 * (size_t)T.hl;
     s_b3[tid][0] = b3[0];
@@ -318,7 +400,7 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  const uint32_t tmem = s_tmem;
+  const uint32_t tmem = __shfl_sync(0xffffffffu, s_tmem, 0);
   const PipeWait wait_bar{&s_abort, P.status};
 
   const uint32_t tp = tmem + (uint32_t)(pipe * T.pipe_stride);
@@ -326,207 +408,193 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   const uint32_t tD = tp + T.col_d, tA = tp + T.col_a, tD3 = tp + T.col_d3, tOnes = tp + T.col_ones;
   const uint32_t tH1 = tOnes - (uint32_t)(T.h1 / 2);                        // layer-2 A operand
   const uint32_t tH2 = T.h2 > 0 ? tOnes - (uint32_t)(T.h2 / 2) : tH1;       // layer-3 A operand
-  // the issuing thread of pipeline p sits in warp 4p + p, so the four issuers use four schedulers
-  const bool leader = (wq == (pipe & 3) && lane == 0);
-  uint64_t* mbar = &bars[1 + pipe];
-  uint32_t phase = 0;
+  // Layers 1 and 2 of pipeline p are issued by its warp p (warp 4p + p of the CTA), layer 3
+  // by its warp p + 1: each scheduler's MMA queue serves one pipeline's layers 1-2 and
+  // another's layer 3, and a pipeline's layer 3 does not queue behind its layer 1.
+  const bool issuer = (wq == (pipe & 3));
+  const bool issuer3 = (wq == ((pipe + 1) & 3));
+  uint64_t* barA = &bars[1 + 2 * pipe];
+  uint64_t* barB = &bars[2 + 2 * pipe];
+  uint32_t phA = 0, phB = 0;
   const int barid = 1 + pipe;
   const uint32_t id1 = idesc_bf16(T.h1), id2 = idesc_bf16(T.h2), id3 = idesc_bf16(T.n3);
   const int s1 = T.k1 / 16, s2 = T.h1 / 16 + 1, s3 = T.hl / 16;
   const int m0 = MP ? T.m0 : 0, m1 = MP ? T.m1 : N;  // this pass's models
   const float vcap = P.vram_cap;
-
   {  // constant ones block: word 0 = (1, 1) feeds the bias hi/lo rows of B2
     uint32_t v[8] = {0x3F803F80u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
     tmem_st_x8(tOnes + lane_off, v);
-    tmem_wait_st();
   }
   wait_bar(&bars[0], 0);  // weights landed
 
-  float thr_s = -INFINITY;
-  uint64_t thr_i = kEmptyIdx;
-  if (MODE == kTcRange) {
-    const CtaTopK tk = topk();
-    thr_s = tk.ls[kcap - 1];
-    thr_i = tk.li[kcap - 1];
-  }
   unsigned int my_count = 0;
 
   const uint64_t n = MODE == kTcRange ? R.len : L.n;
   const uint64_t gpipe = (uint64_t)blockIdx.x * npipes + pipe;
   const uint64_t gstride = (uint64_t)gridDim.x * npipes;
 
-  // range mode: digits of the first candidate, then stepped per tile
-  if (MODE == kTcRange && gpipe * 128 < n) {
-    const uint64_t idx0 = R.base + gpipe * 128 + row;
-    for (int i = 0; i < N; ++i) rows[i * 128 + row] = (uint16_t)(P.off[i] + (int)((idx0 / P.stride[i]) % P.K[i]));
-  }
-
-  auto issue_mma1 = [&](int i) { mma_steps<S1>(s1, tD, tA, desc_s[3 * i + 0], id1, 0u); };
-  auto issue_mma2 = [&](int i) { mma_steps<S2>(s2, tD, tH1, desc_s[3 * i + 1], id2, 0u); };
-  auto issue_mma3 = [&](int i) { mma_steps<S3>(s3, tD3, tH2, desc_s[3 * i + 2], id3, i > m0 ? 1u : 0u); };
-  // fp32 accumulators [0, width) -> ReLU -> bf16 pairs at dst
-  auto epilogue = [&](int width, uint32_t dst) {
-    for (int c0 = 0; c0 < width; c0 += 16) {
-      uint32_t r[16];
-      tmem_ld_x16(tD + lane_off + c0, r);
-      tmem_wait_ld();
-      uint32_t h[8];
-#pragma unroll
-      for (int j = 0; j < 8; ++j) h[j] = relu_bf16x2(r[2 * j], r[2 * j + 1]);
-      tmem_st_x8(dst + lane_off + (c0 >> 1), h);
-    }
+  // UMMA descriptors: every model's image has the same size, so model i's B operands sit
+  // (i - m0) images after model m0's
+  const uint32_t sb1 = smem_base;  // the pass's image starts with model m0's B1
+  const uint32_t sb2 = smem_base + (T.off_b2[0] - T.off_b1[0]);
+  const uint32_t sb3 = smem_base + (T.off_b3[0] - T.off_b1[0]);
+  auto issue_mma1 = [&](int i) {
+    mma_steps<S1>(s1, tD, tA, smem_desc(sb1 + (uint32_t)(i - m0) * T.img_model, 128u, (uint32_t)(T.k1 / 8) * 128u),
+                  id1, 0u);
+  };
+  auto issue_mma2 = [&](int i) {
+    mma_steps<S2>(s2, tD, tH1,
+                  smem_desc(sb2 + (uint32_t)(i - m0) * T.img_model, 128u, (uint32_t)((T.h1 + 16) / 8) * 128u), id2, 0u);
+  };
+  auto issue_mma3 = [&](int i) {
+    mma_steps<S3>(s3, tD3, tH2, smem_desc(sb3 + (uint32_t)(i - m0) * T.img_model, 128u, (uint32_t)(T.hl / 8) * 128u),
+                  id3, i > m0 ? 1u : 0u);
+  };
+  // Every warp waits on the commit's mbarrier itself (suspended until the phase completes).
+  auto await_a = [&]() {
+    if (issuer) wait_bar(barA, phA);
+    phA ^= 1u;
+    named_bar(barid, 128);
+    tc_fence_after();
+  };
+  auto await_b = [&]() {
+    wait_bar(barB, phB);
+    phB ^= 1u;
+    tc_fence_after();
+  };
+  auto publish = [&]() {  // make this thread's tensor-memory stores visible to the issuer
+    tmem_wait_st();
+    tc_fence_before();
+    named_bar(barid, 128);
   };
 
-  bool first_tile = true;
-  for (uint64_t tile = gpipe; tile * 128 < n; tile += gstride) {
+  // ---- A1 rows: [local features | aggregate hi | 1 | aggregate lo] ----
+  // The aggregate words are the same for every model of a tile: they are written with the
+  // tile's first A1 row, and the later models rewrite only the local-feature words (when
+  // the aggregate's position is a compile-time constant).
+  const int awo = AWO >= 0 ? AWO : (T.dle >> 1);
+  auto write_a1 = [&](int i, const uint8_t* dg, bool with_agg, uint4 aw4) {
+    const uint4* src = xw_s + (size_t)(P.off[i] + dg[i * 128 + row]) * (KW >> 2);
+    if (AWO >= 0 && !with_agg) {
+      uint32_t v[AWO > 0 ? AWO : 1];
+#pragma unroll
+      for (int q = 0; q < AWO / 4; ++q) {
+        const uint4 w4 = src[q];
+        v[4 * q + 0] = w4.x; v[4 * q + 1] = w4.y; v[4 * q + 2] = w4.z; v[4 * q + 3] = w4.w;
+      }
+      if constexpr (AWO == 4) tmem_st_x4(tA + lane_off, v);
+      else if constexpr (AWO == 8) tmem_st_x8(tA + lane_off, v);
+      return;
+    }
+    uint32_t v[KW];
+#pragma unroll
+    for (int q = 0; q < KW / 4; ++q) {
+      const uint4 w4 = src[q];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int j = 4 * q + e;
+        const int a = j - awo;
+        const uint32_t x = e == 0 ? w4.x : e == 1 ? w4.y : e == 2 ? w4.z : w4.w;
+        v[j] = a == 0 ? aw4.x : a == 1 ? aw4.y : a == 2 ? aw4.z : a == 3 ? aw4.w : x;
+      }
+    }
+    if constexpr (KW == 8) tmem_st_x8(tA + lane_off, v);
+    else tmem_st_x16(tA + lane_off, v);
+  };
+  // Digits of tile `tile` into buffer dg (range mode: `from`, the previous tile's digits,
+  // stepped by the tile stride) and its first A1 row (model m0) with the aggregate words.
+  auto load_tile = [&](uint64_t tile, uint8_t* dg, const uint8_t* from) {
     const uint64_t t = tile * 128 + row;
-    bool valid = t < n;
-    uint64_t idx = 0;
     if (MODE == kTcRange) {
-      idx = R.base + t;
-      if (!first_tile) {  // add the tile stride to the digits, last model first
+      if (from == nullptr) {
+        const uint64_t idx = R.base + t;
+#pragma unroll (NM > 0 ? NM : 1)
+        for (int i = 0; i < N; ++i) dg[i * 128 + row] = (uint8_t)((idx / P.stride[i]) % P.K[i]);
+      } else {  // add the tile stride to the digits, last model first
         uint32_t carry = 0;
+#pragma unroll (NM > 0 ? NM : 1)
         for (int i = N - 1; i >= 0; --i) {
-          uint32_t d = (uint32_t)rows[i * 128 + row] - (uint32_t)P.off[i] + T.step[i] + carry;
+          uint32_t d = (uint32_t)from[i * 128 + row] + T.step[i] + carry;
           carry = d >= (uint32_t)P.K[i];
           if (carry) d -= (uint32_t)P.K[i];
-          rows[i * 128 + row] = (uint16_t)(P.off[i] + (int)d);
+          dg[i * 128 + row] = (uint8_t)d;
         }
       }
     } else {
-      if (valid) idx = L.idx[t];
-      if (valid && idx >= P.total) {
+      uint64_t idx = t < n ? L.idx[t] : 0;
+      if (t < n && idx >= P.total) {
         atomicOr(P.status, kStatusBadInput);
-        valid = false;
+        idx = 0;  // compute on candidate 0, discard at the end
       }
-      if (!valid) idx = 0;  // compute on candidate 0, discard at the end
-      for (int i = 0; i < N; ++i) rows[i * 128 + row] = (uint16_t)(P.off[i] + digit_of(P, idx, i));
+      for (int i = 0; i < N; ++i) dg[i * 128 + row] = (uint8_t)digit_of(P, idx, i);
     }
-    first_tile = false;
     // aggregate state (fp32, model order) and its bf16 hi/lo words
     float A0 = 0.f, A1 = 0.f, A2 = 0.f;
+#pragma unroll (NM > 0 ? NM : 1)
     for (int i = 0; i < N; ++i) {
-      const float4 d = dem_s[rows[i * 128 + row]];
+      const float4 d = dem_s[P.off[i] + dg[i * 128 + row]];
       A0 += d.x; A1 += d.y; A2 += d.z;
     }
-    uint32_t aw[4];
-    {
+    const float v0 = A0 * P.agg_scale[0], v1 = A1 * P.agg_scale[1], v2 = A2 * P.agg_scale[2];
+    const uint32_t h0 = bf16_bits(v0), h1 = bf16_bits(v1), h2 = bf16_bits(v2);
+    const uint32_t l0 = bf16_bits(v0 - __uint_as_float(h0 << 16));
+    const uint32_t l1 = bf16_bits(v1 - __uint_as_float(h1 << 16));
+    const uint32_t l2 = bf16_bits(v2 - __uint_as_float(h2 << 16));
+    write_a1(m0, dg, true, make_uint4(h0 | (h1 << 16), h2 | (0x3F80u << 16) /* bf16 1.0 */, l0 | (l1 << 16), l2));
+  };
+  // the model-i A1 row of the current tile (aggregate words already in place when AWO >= 0)
+  auto next_a1 = [&](int i, const uint8_t* dg) {
+    if (AWO >= 0) {
+      write_a1(i, dg, false, make_uint4(0u, 0u, 0u, 0u));
+    } else {  // run-time layout: the whole row, aggregate recomputed
+      float A0 = 0.f, A1 = 0.f, A2 = 0.f;
+      for (int j = 0; j < N; ++j) {
+        const float4 d = dem_s[P.off[j] + dg[j * 128 + row]];
+        A0 += d.x; A1 += d.y; A2 += d.z;
+      }
       const float v0 = A0 * P.agg_scale[0], v1 = A1 * P.agg_scale[1], v2 = A2 * P.agg_scale[2];
       const uint32_t h0 = bf16_bits(v0), h1 = bf16_bits(v1), h2 = bf16_bits(v2);
       const uint32_t l0 = bf16_bits(v0 - __uint_as_float(h0 << 16));
       const uint32_t l1 = bf16_bits(v1 - __uint_as_float(h1 << 16));
       const uint32_t l2 = bf16_bits(v2 - __uint_as_float(h2 << 16));
-      aw[0] = h0 | (h1 << 16);
-      aw[1] = h2 | (0x3F80u << 16);  // bf16 1.0
-      aw[2] = l0 | (l1 << 16);
-      aw[3] = l2;
+      write_a1(i, dg, true, make_uint4(h0 | (h1 << 16), h2 | (0x3F80u << 16), l0 | (l1 << 16), l2));
     }
-    // A1 row = option-table words with the aggregate words at word awo (the table holds
-    // zeros there)
-    const int awo = AWO >= 0 ? AWO : (T.dle >> 1);
-    auto word = [&](int j, uint32_t x) -> uint32_t {
-      if (AWO >= 0) return (j >= AWO && j < AWO + 4) ? aw[(j - AWO) & 3] : x;
-      const int a = j - awo;
-      return a == 0 ? aw[0] : a == 1 ? aw[1] : a == 2 ? aw[2] : a == 3 ? aw[3] : x;
-    };
-    auto write_a1 = [&](int i) {
-      const uint4* src = xw_s + (size_t)rows[i * 128 + row] * (KW >> 2);
-      uint32_t v[KW];
-#pragma unroll
-      for (int q = 0; q < KW / 4; ++q) {
-        const uint4 w4 = src[q];
-        v[4 * q + 0] = word(4 * q + 0, w4.x);
-        v[4 * q + 1] = word(4 * q + 1, w4.y);
-        v[4 * q + 2] = word(4 * q + 2, w4.z);
-        v[4 * q + 3] = word(4 * q + 3, w4.w);
-      }
-      if constexpr (KW == 8) tmem_st_x8(tA + lane_off, v);
-      else tmem_st_x16(tA + lane_off, v);
-    };
+  };
 
-    // The issuing thread alone polls the pipeline's mbarrier; the other threads
-    // wait at the named barrier (no issue slots), which the issuer joins once the
-    // MMAs have completed.
-    auto await_mma = [&]() {
-      if (leader) wait_bar(mbar, phase);
-      phase ^= 1u;
-      named_bar(barid, 128);
-      tc_fence_after();
-    };
-    auto publish = [&]() {  // make this thread's tensor-memory stores visible to the issuer
-      tmem_wait_st();
-      tc_fence_before();
-      named_bar(barid, 128);
-    };
-
-    write_a1(m0);
-    publish();
-    for (int i = m0; i < m1; ++i) {
-      if (leader) {
-        tc_fence_after();
-        if (i > m0) issue_mma3(i - 1);
-        issue_mma1(i);
-        mma_commit(mbar);
-      }
-      await_mma();
-      epilogue(T.h1, tH1);  // layer 1 (bias in the constant column)
-      if (T.h2 > 0) {
-        publish();
-        if (leader) {
-          tc_fence_after();
-          issue_mma2(i);
-          mma_commit(mbar);
-        }
-        // layer 1 of model i has completed, so the next A1 goes in while layer 2 runs
-        if (i + 1 < m1) write_a1(i + 1);
-        await_mma();
-        epilogue(T.h2, tH2);  // layer 2 (bias through the ones block)
-      } else if (i + 1 < m1) {
-        write_a1(i + 1);
-      }
-      publish();
-    }
-    if (leader) {
-      tc_fence_after();
-      issue_mma3(m1 - 1);
-      mma_commit(mbar);
-    }
-    await_mma();
-
-    // ---- final epilogue: per-model outputs, constraints, objective ----
-    uint32_t d3[N3 == 16 ? 16 : 32];
-    if constexpr (N3 == 16) {
-      tmem_ld_x16(tD3 + lane_off, d3);
-      tmem_wait_ld();
-    } else if (T.n3 == 16) {
-      uint32_t r16[16];
-      tmem_ld_x16(tD3 + lane_off, r16);
-      tmem_wait_ld();
-#pragma unroll
-      for (int j = 0; j < 16; ++j) d3[j] = r16[j];
+  // ---- objective, constraints and top-k of a finished tile from its layer-3 outputs ----
+  constexpr int D3W = N3 == 16 ? 16 : 32;
+  auto finish_tile = [&](const uint32_t (&d3)[D3W], uint64_t tile_f, const uint8_t* dg) {
+    const uint64_t t = tile_f * 128 + row;
+    bool valid = t < n;
+    uint64_t idx;
+    if (MODE == kTcRange) {
+      idx = R.base + t;
     } else {
-      tmem_ld_x32(tD3 + lane_off, d3);
-      tmem_wait_ld();
+      idx = valid ? L.idx[t] : 0;
+      valid = valid && idx < P.total;
     }
+    float vram = 0.f;  // the candidate's summed VRAM demand (model order, as the aggregate)
+#pragma unroll (NM > 0 ? NM : 1)
+    for (int i = 0; i < N; ++i) vram += dem_s[P.off[i] + dg[i * 128 + row]].y;
     float J = 0.f, pen = 0.f;
     bool sla_ok = true, sla_near = true;
     const int half3 = T.n3 >> 1;  // thr of model i in column i, lat in column half3 + i
+    constexpr int MU = N3 == 16 ? 8 : 16;  // a 16-column layer-3 tile holds at most 8 models
 #pragma unroll
-    for (int i = 0; i < 16; ++i) {
+    for (int i = 0; i < MU; ++i) {
       if (i >= m1) break;
       if (i < m0) continue;
-      const float thr = out_act(P, __uint_as_float(d3[i]) + s_b3[i][0]);
-      const float lat = out_act(P, __uint_as_float(N3 == 16 ? d3[(8 + i) & 15]
-                                                 : half3 == 8 ? d3[(8 + i) & 31] : d3[(16 + i) & 31]) +
-                                   s_b3[i][1]);
+      const float thr = tc_out(P, __uint_as_float(d3[i]) + s_b3[i][0]);
+      const float lat = tc_out(P, __uint_as_float(N3 == 16 ? d3[(8 + i) & 15]
+                                                : half3 == 8 ? d3[(8 + i) & (D3W - 1)] : d3[(16 + i) & (D3W - 1)]) +
+                                  s_b3[i][1]);
       if (MODE == kTcList && valid && L.pred) {
         L.pred[(t * N + i) * 2 + 0] = thr;
         L.pred[(t * N + i) * 2 + 1] = lat;
       }
       if (UT) {  // Eq. 3 utility, floors f >= tau
         float f;
-        J += util_term(P, i, rows[i * 128 + row], thr, &f);
+        J += util_term(P, i, P.off[i] + dg[i * 128 + row], thr, &f);
         const float tau = P.u_tau[i];
         sla_ok = sla_ok && (f >= tau);
         sla_near = sla_near && (f >= tau - 2e-2f * fmaxf(fabsf(tau), fabsf(f)));
@@ -550,9 +618,9 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     }
     if (MP && !T.pass_last) {  // (uniform) hand the partial objective to the next pass
       if (t < n) T.partial[t] = make_float4(J, pen, __uint_as_float((sla_ok ? 1u : 0u) | (sla_near ? 2u : 0u)), 0.f);
-      continue;
+      return;
     }
-    bool feas = valid && A1 <= vcap;
+    bool feas = valid && vram <= vcap;
     bool cand = feas;
     if (!UT && P.objective == MF_OBJ_SOFT_LAT) {
       J = fmaf(-P.soft_penalty, pen, J);
@@ -568,19 +636,98 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
       }
     } else {
       my_count += feas ? 1u : 0u;
-      const bool push = cand && precedes(J, idx, thr_s, thr_i);
       const CtaTopK tk = topk();
+      const bool push = cand && precedes(J, idx, tk.ls[kcap - 1], tk.li[kcap - 1]);
       if (push) {
         const int pos = atomicAdd(tk.qn, 1);
         tk.qs[pos] = J;
         tk.qi[pos] = idx;
       }
-      if (named_bar_or(barid, 128, push)) {
-        tc_topk_merge(tk, row, barid);
-        thr_s = tk.ls[kcap - 1];
-        thr_i = tk.li[kcap - 1];
-      }
+      if (named_bar_or(barid, 128, push)) tc_topk_merge(tk, row, barid);
     }
+  };
+  auto load_d3 = [&](uint32_t (&d3)[D3W]) {
+    if constexpr (N3 == 16) {
+      tmem_ld_x16(tD3 + lane_off, d3);
+    } else if (T.n3 == 16) {
+      uint32_t r16[16];
+      tmem_ld_x16(tD3 + lane_off, r16);
+      tmem_wait_ld();
+#pragma unroll
+      for (int j = 0; j < 16; ++j) d3[j] = r16[j];
+    } else {
+      tmem_ld_x32(tD3 + lane_off, d3);
+    }
+    tmem_wait_ld();
+  };
+
+  uint64_t tile = gpipe;
+  int buf = 0;
+  if (tile * 128 < n) load_tile(tile, digits, nullptr);
+  publish();  // ones block and the first A1
+
+  // the previous tile is finished once its last layer 3 (issued in this tile's first
+  // round A) has landed
+  bool pending = false;
+  uint32_t d3[D3W];
+
+  for (; tile * 128 < n; tile += gstride) {
+    uint8_t* dg = digits + buf * (MF_MAX_MODELS * 128);
+    uint8_t* dg_p = digits + (buf ^ 1) * (MF_MAX_MODELS * 128);
+    const bool has_next = (tile + gstride) * 128 < n;
+#pragma unroll (NM > 0 ? NM : 1)
+    for (int i = m0; i < m1; ++i) {
+      const bool l3 = i > m0 || pending;
+      // ---- round A: layer 1 of model i, layer 3 of the model before ----
+      if (issuer) {
+        tc_fence_after();
+        issue_mma1(i);
+        mma_commit_warp(barA);
+      } else if (issuer3 && l3) {
+        tc_fence_after();
+        issue_mma3(i > m0 ? i - 1 : m1 - 1);
+        mma_commit_warp(barB);
+      }
+      await_a();
+      hidden_epilogue<(S2 > 0 ? (S2 - 1) * 16 : 0)>(T.h1, tD + lane_off, tH1 + lane_off, [&]() {
+        if (l3) {
+          await_b();
+          if (i == m0) load_d3(d3);  // the previous tile's outputs, before layer 3 restarts
+        }
+      });
+      if (T.h2 == 0) {  // one hidden layer: no round B
+        if (i + 1 < m1) next_a1(i + 1, dg);
+        else if (has_next) load_tile(tile + gstride, dg_p, dg);
+        publish();
+        if (i == m0 && pending) finish_tile(d3, tile - gstride, dg_p);
+        continue;
+      }
+      publish();
+      // ---- round B: layer 2 of model i ----
+      if (issuer) {
+        tc_fence_after();
+        issue_mma2(i);
+        mma_commit_warp(barA);
+      }
+      if (i == m0 && pending) finish_tile(d3, tile - gstride, dg_p);
+      if (i + 1 < m1) next_a1(i + 1, dg);
+      else if (has_next) load_tile(tile + gstride, dg_p, dg);  // next tile: digits, aggregate, A1
+      await_a();
+      hidden_epilogue<(S3 > 0 ? S3 * 16 : 0)>(T.h2, tD + lane_off, tH2 + lane_off, []() {});
+      publish();
+    }
+    pending = true;
+    buf ^= 1;
+  }
+  if (pending) {  // the last tile's last layer 3
+    if (issuer3) {
+      tc_fence_after();
+      issue_mma3(m1 - 1);
+      mma_commit_warp(barB);
+    }
+    await_b();
+    load_d3(d3);
+    finish_tile(d3, tile - gstride, digits + (buf ^ 1) * (MF_MAX_MODELS * 128));
   }
 
   if (MODE == kTcRange && (!MP || T.pass_last)) {
@@ -646,11 +793,10 @@ void layout_smem(const Params& P, TcArgs& T, int kcap) {
   uint32_t o = round_up((int)T.img_bytes, 1024);
   T.sm_xw = o; o += round_up(sumK * T.kw * 4, 16);
   T.sm_dem = o; o += sumK * 16;
-  T.sm_rows = o; o += T.pipes * MF_MAX_MODELS * 128 * 2;
-  T.sm_desc = o; o += 8 * 3 * MF_MAX_MODELS;
+  T.sm_rows = o; o += T.pipes * 2 * MF_MAX_MODELS * 128;  // byte digits of two tiles per pipeline
   T.sm_topk = o; o += kcap > 0 ? (uint32_t)(T.pipes * topk_bytes_pipe(kcap)) : 0u;
   o = round_up((int)o, 16);
-  T.sm_bar = o; o += 8 * (kTcMaxPipes + 1);
+  T.sm_bar = o; o += 8 * (1 + 2 * kTcMaxPipes);
   T.sm_total = o;
   T.kcap = kcap;
 }
@@ -663,25 +809,29 @@ using TcFn = void (*)(const Params, const TcArgs, const RangeArgs, const TcList)
 // Instantiations: the two benchmark shapes (d_L 8, 64-64 and d_L 16, 128-128, up to 8
 // models) with all counts fixed at compile time, and a run-time fallback per A1 row width.
 template <int MODE, bool MP, bool UT>
-TcFn tc_kernel_mode(const TcArgs& T) {
+TcFn tc_kernel_mode(const TcArgs& T, int n_models) {
   // S1 = k1 / 16, S2 = h1 / 16 + 1 (the b2 step), S3 = hl / 16
-  if (T.kw == 8 && T.dle == 8 && T.h1 == 64 && T.h2 == 64 && T.n3 == 16)
-    return k_score_tc<MODE, 8, 4, 1, 5, 4, 16, MP, UT>;
+  if (T.kw == 8 && T.dle == 8 && T.h1 == 64 && T.h2 == 64 && T.n3 == 16) {
+    if constexpr (MODE == kTcRange && !MP && !UT) {
+      if (n_models == 6) return k_score_tc<MODE, 8, 4, 1, 5, 4, 16, MP, UT, 6>;  // the 24^6 workload's shape
+    }
+    return k_score_tc<MODE, 8, 4, 1, 5, 4, 16, MP, UT, 0>;
+  }
   if (T.kw == 16 && T.dle == 16 && T.h1 == 128 && T.h2 == 128 && T.n3 == 16)
-    return k_score_tc<MODE, 16, 8, 2, 9, 8, 16, MP, UT>;
-  if (T.kw == 8) return k_score_tc<MODE, 8, -1, 0, 0, 0, 0, MP, UT>;
-  return k_score_tc<MODE, 16, -1, 0, 0, 0, 0, MP, UT>;
+    return k_score_tc<MODE, 16, 8, 2, 9, 8, 16, MP, UT, 0>;
+  if (T.kw == 8) return k_score_tc<MODE, 8, -1, 0, 0, 0, 0, MP, UT, 0>;
+  return k_score_tc<MODE, 16, -1, 0, 0, 0, 0, MP, UT, 0>;
 }
 
 template <bool UT>
-TcFn tc_kernel_ut(int mode, const TcArgs& T) {
+TcFn tc_kernel_ut(int mode, const TcArgs& T, int n) {
   if (T.npasses > 1)
-    return mode == kTcRange ? tc_kernel_mode<kTcRange, true, UT>(T) : tc_kernel_mode<kTcList, true, UT>(T);
-  return mode == kTcRange ? tc_kernel_mode<kTcRange, false, UT>(T) : tc_kernel_mode<kTcList, false, UT>(T);
+    return mode == kTcRange ? tc_kernel_mode<kTcRange, true, UT>(T, n) : tc_kernel_mode<kTcList, true, UT>(T, n);
+  return mode == kTcRange ? tc_kernel_mode<kTcRange, false, UT>(T, n) : tc_kernel_mode<kTcList, false, UT>(T, n);
 }
 
-TcFn tc_kernel(int mode, const TcArgs& T, bool util) {
-  return util ? tc_kernel_ut<true>(mode, T) : tc_kernel_ut<false>(mode, T);
+TcFn tc_kernel(int mode, const TcArgs& T, bool util, int n) {
+  return util ? tc_kernel_ut<true>(mode, T, n) : tc_kernel_ut<false>(mode, T, n);
 }
 constexpr uint32_t kSmemFloor = 120 * 1024;          // keeps one CTA (one TMEM owner) per SM
 
@@ -809,6 +959,7 @@ mf_status tc_prepare(mf_ctx* c) {
     }
     T.off_b3[i] = (uint32_t)img.size();
     img.resize(img.size() + b3_bytes, 0);
+    T.img_model = (uint32_t)(b1_bytes + b2_bytes + b3_bytes);  // the kernel steps descriptors by it
     for (int k = 0; k < hl; ++k) {
       put(T.off_b3[i], i, k, k3, W3[k]);
       put(T.off_b3[i], T.n3 / 2 + i, k, k3, W3[hl + k]);
@@ -854,8 +1005,8 @@ mf_status tc_prepare(mf_ctx* c) {
   T.img = base;
   T.xw = reinterpret_cast<const uint32_t*>(base + o_xw);
   for (int u = 0; u < 2; ++u) {
-    MF_CUDA(cudaFuncSetAttribute(tc_kernel(kTcRange, T, u), cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit));
-    MF_CUDA(cudaFuncSetAttribute(tc_kernel(kTcList, T, u), cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit));
+    MF_CUDA(cudaFuncSetAttribute(tc_kernel(kTcRange, T, u, P.n_models), cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit));
+    MF_CUDA(cudaFuncSetAttribute(tc_kernel(kTcList, T, u, P.n_models), cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit));
   }
   layout_smem(P, T, 0);
   if (T.sm_total > kSmemLimit) {
@@ -896,7 +1047,7 @@ mf_status tc_search_chunk(mf_ctx* c, const RangeArgs& a, cudaStream_t s, int* nl
     r.first = a.first && b == 0;
     for (int p = 0; p < T.npasses; ++p) {
       set_pass(T, p, partial);
-      tc_kernel(kTcRange, T, c->P.objective == MF_OBJ_UTILITY)<<<c->num_sms, T.pipes * 128, smem, s>>>(c->P, T, r, L);
+      tc_kernel(kTcRange, T, c->P.objective == MF_OBJ_UTILITY, c->P.n_models)<<<c->num_sms, T.pipes * 128, smem, s>>>(c->P, T, r, L);
       MF_CUDA(cudaGetLastError());
       ++launches;
     }
@@ -926,7 +1077,7 @@ mf_status tc_score_list(mf_ctx* c, const uint64_t* idx, uint64_t n, float* score
     TcList L{idx + b, m, score + b, feas ? feas + b : nullptr, pred ? pred + b * N * 2 : nullptr};
     for (int p = 0; p < T.npasses; ++p) {
       set_pass(T, p, partial);
-      tc_kernel(kTcList, T, c->P.objective == MF_OBJ_UTILITY)<<<(unsigned)grid, T.pipes * 128, smem, s>>>(c->P, T, R, L);
+      tc_kernel(kTcList, T, c->P.objective == MF_OBJ_UTILITY, c->P.n_models)<<<(unsigned)grid, T.pipes * 128, smem, s>>>(c->P, T, R, L);
       MF_CUDA(cudaGetLastError());
     }
   }

@@ -48,7 +48,8 @@ struct TcArgs {
   int32_t k1, kw, h1, h2, hl, n3, dle;
   uint32_t off_b1[MF_MAX_MODELS], off_b2[MF_MAX_MODELS], off_b3[MF_MAX_MODELS];  // bytes in img
   int32_t pipes, col_d, col_h, col_ones, col_a, col_d3, pipe_stride;  // TMEM columns
-  uint32_t sm_xw, sm_dem, sm_rows, sm_desc, sm_topk, sm_bar, sm_total;  // shared-memory byte offsets
+  uint32_t sm_xw, sm_dem, sm_rows, sm_topk, sm_bar, sm_total;  // shared-memory byte offsets
+  uint32_t img_model;                 // bytes of one model's B1 + B2 + B3 images
   int32_t kcap;                       // per-pipeline list length the layout was sized for
   uint32_t step[MF_MAX_MODELS];       // mixed-radix digits of the per-tile index stride (range mode)
   // models whose weights do not fit shared memory together run in passes of consecutive
