@@ -269,3 +269,63 @@ def test_paper_ga_is_deterministic_and_seeded(oracle_mod):
     assert a[0] == o.fc_ga_run(fc, g, 11)[0] and np.array_equal(a[1], o.fc_ga_run(fc, g, 11)[1])
     outs = {tuple(o.fc_ga_run(fc, g, s)[1]) for s in range(11, 19)}
     assert len(outs) > 1  # three generations do not always reach the same configuration
+
+
+# ---------------------------------------------------------------------------
+# The paper GA's loop (Sec. IV-C), pinned by pieces that have their own pins:
+# the counter-based generator (published SplitMix64 outputs), the integer draw
+# rule (multiply-shift of the top 32 bits) and the fixed-context table.
+# ---------------------------------------------------------------------------
+def _all_feasible_fc(prob, seed):
+    fc = W.fc_scenario(prob, seed)
+    return dict(fc, tau=np.full(len(prob["n_options"]), -1e6, np.float32))
+
+
+def test_paper_ga_of_one_generation_returns_the_best_initial_draw(oracle_mod):
+    """gens = 1: the initial population alone, individual c drawing gene i as
+    floor(hi32(rng(seed, 0, c, init, i)) * K_i / 2^32); without repair and with no
+    floor or VRAM limit in reach the result is the individual with the largest
+    sum of table utilities (lowest slot among equals)."""
+    prob = W.paper_scale()
+    prob = dict(prob, vram_cap=1e9)
+    o = oracle_mod.Oracle(prob)
+    fc = _all_feasible_fc(prob, 4)
+    _, _, ok, u = o.fc_local(fc)
+    assert ok.all()
+    K = [int(k) for k in prob["n_options"]]
+    off = np.concatenate([[0], np.cumsum(K)])
+    g = dict(W.PAPER_GA_PARAMS, gens=1, repair=0, pop=37)
+    for seed in (1000, 1001):
+        pop = np.array([[((oracle_mod.rng(seed, 0, c, 0, i) >> 32) * K[i]) >> 32 for i in range(len(K))]
+                        for c in range(g["pop"])])
+        fit = np.array([sum(u[off[i] + pop[c, i]] for i in range(len(K))) for c in range(g["pop"])])
+        e = int(np.argmax(fit))
+        J, genome = o.fc_ga_run(fc, g, seed)
+        assert list(genome) == list(pop[e])
+        assert J == pytest.approx(fit[e], rel=0, abs=1e-12)
+
+
+def test_paper_ga_without_mutation_or_crossover_keeps_the_initial_genes(oracle_mod):
+    """p_m = 0 and p_c = 0: every child copies a tournament winner, so on one model
+    with two options the decision over any number of generations is the best option
+    present in the initial population."""
+    prob = W.make_problem([2], 8, 16, 0, 41, 1e9)
+    o = oracle_mod.Oracle(prob)
+    fc = _all_feasible_fc(prob, 41)
+    _, _, ok, u = o.fc_local(fc)
+    assert ok.all() and u[0] != u[1]
+    seen = set()
+    for seed in range(300):
+        g0 = dict(W.PAPER_GA_PARAMS, pop=2, gens=1, repair=0, mutation_p=0.0, crossover_p=0.0)
+        init = [((oracle_mod.rng(seed, 0, c, 0, 0) >> 32) * 2) >> 32 for c in range(2)]
+        kind = tuple(sorted(set(init)))
+        if kind in seen:
+            continue
+        seen.add(kind)
+        expect = max(kind, key=lambda k: u[k])
+        for gens in range(1, 7):
+            J, genome = o.fc_ga_run(fc, dict(g0, gens=gens), seed)
+            assert genome[0] == expect and J == pytest.approx(u[expect], rel=0, abs=1e-12)
+        if len(seen) == 3:
+            break
+    assert seen == {(0,), (1,), (0, 1)}

@@ -168,3 +168,88 @@ def test_integer_landscape_is_exact_in_any_order(oracle_mod, opts, seed, cap):
     s, f, pred, _ = o.score_list(idx, with_pred=True)
     assert np.all(pred == np.round(pred))
     assert f.any() and np.all(2 * s[f] == np.round(2 * s[f]))  # soft penalty 0.5: halves
+
+
+# ---------------------------------------------------------------------------
+# The GA loop (Sec. IV-C): which population is evaluated how often, and which
+# individual is returned.  Each pin composes only separately pinned pieces (the
+# initial population, the step operator, the predictor and objective).
+# ---------------------------------------------------------------------------
+def _fitness(o, pop):
+    return np.array([o.score_digits(row)[0] for row in pop])
+
+
+def test_ga_run_of_one_generation_returns_the_best_initial_individual(oracle_mod):
+    """gens = 1 evaluates the initial population once and returns its fittest
+    individual (lowest slot among equals), with no generation step."""
+    p = W.random_small(21, 3, max_options=6, h1=16, vram_cap=30.0)
+    o = oracle_mod.Oracle(p)
+    for seed in (3, 4, 5):
+        g = _ga(pop=48, gens=1)
+        pop0 = o.ga_init(g, seed)
+        fit = _fitness(o, pop0)
+        e = int(np.argmax(fit))  # first maximum: the lowest slot among equals
+        J, genome = o.ga_run(g, seed)
+        assert J == fit[e]
+        assert list(genome) == list(pop0[e])
+
+
+@pytest.mark.parametrize("gens", [2, 3, 5])
+def test_ga_run_is_the_initial_population_then_gens_minus_one_steps(oracle_mod, gens):
+    """gens evaluations: the initial population, then a step with generation index
+    0, 1, ..., gens - 2, each step taking the fitness of the population it breeds
+    from; the result is the fittest individual of the last evaluated population."""
+    p = W.random_small(22, 4, max_options=5, h1=16, vram_cap=40.0)
+    o = oracle_mod.Oracle(p)
+    g = _ga(pop=40, gens=gens)
+    seed = 77
+    pop = o.ga_init(g, seed)
+    for gen in range(gens - 1):
+        pop = o.ga_step(g, seed, gen, pop, _fitness(o, pop))
+    fit = _fitness(o, pop)
+    e = int(np.argmax(fit))
+    J, genome = o.ga_run(g, seed)
+    assert J == fit[e]
+    assert list(genome) == list(pop[e])
+
+
+def _two_option_problem(oracle_mod, seed):
+    """One model with two options, both feasible (no SLA or VRAM limit in reach)."""
+    p = W.make_problem([2], 8, 16, 0, seed, 1e9)
+    p["sla"] = np.array([1e9], np.float32)
+    o = oracle_mod.Oracle(p)
+    J = [o.score_digits([k])[0] for k in (0, 1)]
+    assert J[0] != J[1] and np.isfinite(J).all()
+    return o, J
+
+
+def test_ga_without_mutation_keeps_to_the_genes_of_the_initial_population(oracle_mod):
+    """With mutation off, crossover and selection can only recombine genes already
+    present: on one model with two options a population that starts without the
+    better option never finds it, and one that starts with it returns it from the
+    first generation on (elitism keeps it)."""
+    o, J = _two_option_problem(oracle_mod, 31)
+    best = int(np.argmax(J))
+    seen = set()
+    for seed in range(200):
+        g = _ga(pop=2, gens=1, mutation_p=0.0, tournament=2)
+        has_best = best in set(o.ga_init(g, seed)[:, 0].tolist())
+        if has_best in seen:
+            continue
+        seen.add(has_best)
+        expect = best if has_best else 1 - best  # two options: without the best, only the other
+        for gens in range(1, 7):
+            Jr, genome = o.ga_run(_ga(pop=2, gens=gens, mutation_p=0.0, tournament=2), seed)
+            assert genome[0] == expect and Jr == J[expect]
+        if len(seen) == 2:
+            break
+    assert seen == {True, False}
+
+
+def test_ga_with_elitism_never_loses_its_best(oracle_mod):
+    """One elite: the returned fitness does not decrease with the number of
+    generations for a fixed seed."""
+    p = W.random_small(23, 4, max_options=6, h1=16, vram_cap=35.0)
+    o = oracle_mod.Oracle(p)
+    Js = [o.ga_run(_ga(pop=24, gens=g), 9)[0] for g in range(1, 9)]
+    assert all(b >= a for a, b in zip(Js, Js[1:]))
