@@ -86,6 +86,10 @@ __device__ __forceinline__ void named_bar(int id, int nthreads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
 
+__device__ __forceinline__ void named_arrive(int id, int nthreads) {
+  asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+
 // OR of `pred` over the threads of a named barrier (also a barrier).
 __device__ __forceinline__ bool named_bar_or(int id, int nthreads, bool pred) {
   uint32_t r;
@@ -217,6 +221,24 @@ struct PipeWait {
   }
 };
 
+// A wait that ignores an earlier give-up, for the work this CTA itself has in flight
+// (its MMAs, its weight copy) before the tensor memory is freed; bounded all the same.
+__device__ __noinline__ void mbar_wait_drain(uint64_t* bar, uint32_t parity, uint32_t* status) {
+  for (uint32_t n = 0; n < kWaitLimit; ++n)
+    if (mbar_try_wait(bar, parity)) return;
+  atomicOr(status, kStatusTimeout);
+}
+
+// The planted wait of the timeout test: a barrier that nothing arrives on, `polls`
+// suspended tries; giving up flags the status word and sets the CTA's give-up flag.
+__device__ __noinline__ void mbar_wait_test(uint64_t* never, uint32_t polls, volatile int* abort,
+                                            uint32_t* status) {
+  for (uint32_t n = 0; n < polls; ++n)
+    if (mbar_try_wait(never, 0)) return;
+  *abort = 1;
+  atomicOr(status, kStatusTimeout);
+}
+
 // The predictor's output unit; the sigmoid out of line keeps the scorer's loop small.
 __device__ __noinline__ float tc_sigmoid(float v) { return 1.f / (1.f + expf(-v)); }
 __device__ __forceinline__ float tc_out(const Params& P, float v) {
@@ -255,11 +277,13 @@ __device__ __forceinline__ void mma_steps(int steps, uint32_t d_tmem, uint32_t a
 }
 
 // Hidden epilogue: fp32 accumulators [0, width) at `src` -> ReLU -> bf16 pairs at `dst`.
-// 64 columns are loaded before one wait.  `before_store` runs once, after the first
-// piece's loads and conversions and before its stores (round A waits there for the
+// 64 columns are loaded before one wait.  `after_load` runs once the last accumulator
+// column is in registers (the accumulator columns are then free for the next layer);
+// `before_store` runs once, before the first stores (round A waits there for the
 // previous model's layer 3, which reads the same tensor-memory columns).
-template <int W, class F>
-__device__ __forceinline__ void hidden_epilogue(int width, uint32_t src, uint32_t dst, F before_store) {
+template <int W, class FL, class FS>
+__device__ __forceinline__ void hidden_epilogue(int width, uint32_t src, uint32_t dst, FL after_load,
+                                                FS before_store) {
   if constexpr (W > 0 && W % 64 == 0) {
 #pragma unroll 1
     for (int c0 = 0; c0 < W; c0 += 64) {
@@ -267,6 +291,7 @@ __device__ __forceinline__ void hidden_epilogue(int width, uint32_t src, uint32_
       tmem_ld_x32(src + c0, a);
       tmem_ld_x32(src + c0 + 32, b);
       tmem_wait_ld();
+      if (c0 + 64 == W) after_load();
       uint32_t h[16], g[16];
 #pragma unroll
       for (int j = 0; j < 16; ++j) h[j] = relu_bf16x2(a[2 * j], a[2 * j + 1]);
@@ -281,6 +306,7 @@ __device__ __forceinline__ void hidden_epilogue(int width, uint32_t src, uint32_
       uint32_t a[32];
       tmem_ld_x32(src + c0, a);
       tmem_wait_ld();
+      if (c0 + 32 >= width) after_load();
       uint32_t h[16];
 #pragma unroll
       for (int j = 0; j < 16; ++j) h[j] = relu_bf16x2(a[2 * j], a[2 * j + 1]);
@@ -340,6 +366,8 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   if (tid == 0) {
     s_abort = 0;
     for (int j = 0; j < 1 + 2 * npipes; ++j) mbar_init(&bars[j], 1);
+    mbar_init(&bars[1 + 2 * npipes], 1);           // the timeout test's barrier: nothing arrives
+    mbar_init(&bars[2 + 2 * npipes], 2 * npipes);  // drain: one commit per issuing warp
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 0) {
@@ -417,6 +445,7 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   uint64_t* barB = &bars[2 + 2 * pipe];
   uint32_t phA = 0, phB = 0;
   const int barid = 1 + pipe;
+  const int barid_d = 1 + npipes + pipe;  // "accumulators read": the issuing warp syncs, the rest arrive
   const uint32_t id1 = idesc_bf16(T.h1), id2 = idesc_bf16(T.h2), id3 = idesc_bf16(T.n3);
   const int s1 = T.k1 / 16, s2 = T.h1 / 16 + 1, s3 = T.hl / 16;
   const int m0 = MP ? T.m0 : 0, m1 = MP ? T.m1 : N;  // this pass's models
@@ -425,6 +454,7 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     uint32_t v[8] = {0x3F803F80u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
     tmem_st_x8(tOnes + lane_off, v);
   }
+  if (P.wait_test) mbar_wait_test(&bars[1 + 2 * npipes], P.wait_test, &s_abort, P.status);
   wait_bar(&bars[0], 0);  // weights landed
 
   unsigned int my_count = 0;
@@ -466,6 +496,20 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     tmem_wait_st();
     tc_fence_before();
     named_bar(barid, 128);
+  };
+  // The accumulators have been read and the next A1 row written: the issuing warp starts
+  // the next layer 1 while the others go on converting.
+  auto issue_next_l1 = [&](int inext) {
+    tmem_wait_st();
+    tc_fence_before();
+    if (issuer) {
+      named_bar(barid_d, 128);
+      tc_fence_after();
+      issue_mma1(inext);
+      mma_commit_warp(barA);
+    } else {
+      named_arrive(barid_d, 128);
+    }
   };
 
   // ---- A1 rows: [local features | aggregate hi | 1 | aggregate lo] ----
@@ -665,6 +709,11 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   int buf = 0;
   if (tile * 128 < n) load_tile(tile, digits, nullptr);
   publish();  // ones block and the first A1
+  if (tile * 128 < n && issuer) {  // the first layer 1; every later one starts in the round before
+    tc_fence_after();
+    issue_mma1(m0);
+    mma_commit_warp(barA);
+  }
 
   // the previous tile is finished once its last layer 3 (issued in this tile's first
   // round A) has landed
@@ -678,28 +727,27 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
 #pragma unroll (NM > 0 ? NM : 1)
     for (int i = m0; i < m1; ++i) {
       const bool l3 = i > m0 || pending;
-      // ---- round A: layer 1 of model i, layer 3 of the model before ----
-      if (issuer) {
-        tc_fence_after();
-        issue_mma1(i);
-        mma_commit_warp(barA);
-      } else if (issuer3 && l3) {
+      const bool next_l1 = i + 1 < m1 || has_next;
+      const int inext = i + 1 < m1 ? i + 1 : m0;
+      // ---- round A: layer 1 of model i (already issued), layer 3 of the model before ----
+      if (issuer3 && l3) {
         tc_fence_after();
         issue_mma3(i > m0 ? i - 1 : m1 - 1);
         mma_commit_warp(barB);
       }
       await_a();
-      hidden_epilogue<(S2 > 0 ? (S2 - 1) * 16 : 0)>(T.h1, tD + lane_off, tH1 + lane_off, [&]() {
+      hidden_epilogue<(S2 > 0 ? (S2 - 1) * 16 : 0)>(T.h1, tD + lane_off, tH1 + lane_off, []() {}, [&]() {
         if (l3) {
           await_b();
           if (i == m0) load_d3(d3);  // the previous tile's outputs, before layer 3 restarts
         }
       });
       if (T.h2 == 0) {  // one hidden layer: no round B
+        if (i == m0 && pending) finish_tile(d3, tile - gstride, dg_p);
         if (i + 1 < m1) next_a1(i + 1, dg);
         else if (has_next) load_tile(tile + gstride, dg_p, dg);
+        if (next_l1) issue_next_l1(inext);
         publish();
-        if (i == m0 && pending) finish_tile(d3, tile - gstride, dg_p);
         continue;
       }
       publish();
@@ -713,7 +761,12 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
       if (i + 1 < m1) next_a1(i + 1, dg);
       else if (has_next) load_tile(tile + gstride, dg_p, dg);  // next tile: digits, aggregate, A1
       await_a();
-      hidden_epilogue<(S3 > 0 ? S3 * 16 : 0)>(T.h2, tD + lane_off, tH2 + lane_off, []() {});
+      hidden_epilogue<(S3 > 0 ? S3 * 16 : 0)>(
+          T.h2, tD + lane_off, tH2 + lane_off,
+          [&]() {
+            if (next_l1) issue_next_l1(inext);
+          },
+          []() {});
       publish();
     }
     pending = true;
@@ -742,6 +795,12 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
     if (lane == 0 && c) atomicAdd(R.count, (unsigned long long)c);
   }
+  // Nothing of this CTA may still run when its tensor memory is freed: each issuing warp
+  // commits its MMAs to the drain barrier, and everyone waits for them and for the weight
+  // copy (after a wait that gave up, these are the only waits still made).
+  if (issuer || issuer3) mma_commit_warp(&bars[2 + 2 * npipes]);
+  mbar_wait_drain(&bars[2 + 2 * npipes], 0, P.status);
+  mbar_wait_drain(&bars[0], 0, P.status);
   tc_fence_before();
   __syncthreads();
   if (warp == 0) {
@@ -796,7 +855,7 @@ void layout_smem(const Params& P, TcArgs& T, int kcap) {
   T.sm_rows = o; o += T.pipes * 2 * MF_MAX_MODELS * 128;  // byte digits of two tiles per pipeline
   T.sm_topk = o; o += kcap > 0 ? (uint32_t)(T.pipes * topk_bytes_pipe(kcap)) : 0u;
   o = round_up((int)o, 16);
-  T.sm_bar = o; o += 8 * (1 + 2 * kTcMaxPipes);
+  T.sm_bar = o; o += 8 * (3 + 2 * kTcMaxPipes);
   T.sm_total = o;
   T.kcap = kcap;
 }
