@@ -319,8 +319,13 @@ mf_status mf_get_stats(const mf_ctx *ctx, mf_stats *out);
  * MF_NOALLOC_SCRATCH_BYTES.  At most MF_NOALLOC_MAX_CTAS CTAs are launched.
  *
  * The first call on a device looks up the array's device address (once per
- * device, with that device current); make that first call before any stream
- * capture.  Every call on a device shares the one array and overwrites it
+ * device, with that device current), and that lookup is what makes the runtime
+ * load the library's module and reserve the array on the device: a caller whose
+ * memory pool will claim the device's memory makes the first call before the pool
+ * does, and before any stream capture.  A cudaDeviceReset releases the array but
+ * not the cached address, so after resetting a device do not call this entry point
+ * on it again.  A call that fails after it has queued work waits for that work
+ * before returning.  Every call on a device shares the one array and overwrites it
  * (what must start at zero is cleared at the start of each call), so calls
  * that overlap on the GPU -- from several host threads or streams -- race and
  * must be serialised by the caller.  Synchronous: returns after `out` is filled. */
@@ -334,6 +339,18 @@ mf_status mf_search_exhaustive_noalloc(const mf_problem *p, int32_t k, uint64_t 
 /* Synchronise `stream`, then return MF_EDEVICE if any asynchronous call since the
  * last check saw an invalid index or gene (and clear that flag), else MF_OK. */
 mf_status mf_check_device_status(mf_ctx *ctx, void *stream);
+
+/* For tests of the failure path of the bounded device waits; the paper has no
+ * counterpart.  With polls > 0, every later launch on `ctx` of a kernel that waits
+ * on the device (the tensor-core scorer behind mf_search_* / mf_score_batch in
+ * MF_BF16, and the single-kernel GA of mf_ga_run) first waits on a flag that
+ * nothing sets, giving up after `polls` polls (about a millisecond each in the
+ * scorer, a few nanoseconds in the GA kernel).  The kernel then flags the context's
+ * device status and runs to its end without waiting again, except for its own
+ * MMAs and weight copies in flight, which it always drains before it frees its
+ * tensor memory; the call returns MF_ETIMEOUT and its results are undefined.  The
+ * context stays usable: polls = 0 restores normal operation.  MF_EINVAL: ctx NULL. */
+mf_status mf_debug_wait_test(mf_ctx *ctx, uint32_t polls);
 
 #ifdef __cplusplus
 }

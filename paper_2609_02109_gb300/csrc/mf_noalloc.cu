@@ -6,9 +6,15 @@
 // mf_search_exhaustive_noalloc runs the exact fp32 exhaustive search with all
 // of its device memory (the problem's tables and weights, the per-CTA running
 // top-k lists, the merge buffers, the feasible counter and the status word) in
-// one file-scope __device__ array of fixed size.  Every GPU that loads the
-// library holds that array until the process exits.  The entry point calls no
-// cudaMalloc, cudaFree or other allocating routine.
+// one file-scope __device__ array of fixed size.  The runtime loads the module that
+// holds the array lazily, so the array is reserved on a device by the first call
+// there (its cudaGetSymbolAddress loads the module): a caller whose pool will claim
+// the device's memory makes that first call before the pool does, and before any
+// stream capture.  From then on the device holds the array until the process exits,
+// and the entry point calls no cudaMalloc, cudaFree or other allocating routine.  A
+// cudaDeviceReset releases the array while the address looked up at the first call
+// stays cached, so a process that resets a device must not call this entry point on
+// that device again.
 #include <mutex>
 
 #include "mf_internal.cuh"
@@ -176,6 +182,16 @@ extern "C" mf_status mf_search_exhaustive_noalloc(const mf_problem* p, int32_t k
   mf_status s0 = scratch_address(dev, &base);
   if (s0 != MF_OK) return s0;
   cudaStream_t s = (cudaStream_t)stream;
+  // From the first enqueue on, a failing return first waits for the work already on the
+  // stream, so no copy or kernel of this call is still using the shared array when the
+  // caller's next call starts.
+  struct Drain {
+    cudaStream_t s;
+    bool armed = true;
+    ~Drain() {
+      if (armed) cudaStreamSynchronize(s);
+    }
+  } drain{s};
 
   // inputs: the caller's host arrays into the scratch, then the internal layouts
   MF_CUDA(cudaMemcpyAsync(base + o_x, p->local_feats, b_x, cudaMemcpyHostToDevice, s));
@@ -226,6 +242,7 @@ extern "C" mf_status mf_search_exhaustive_noalloc(const mf_problem* p, int32_t k
   if (out->topk_score)
     MF_CUDA(cudaMemcpyAsync(out->topk_score, base + o_fs, sizeof(float) * k, cudaMemcpyDeviceToHost, s));
   MF_CUDA(cudaStreamSynchronize(s));
+  drain.armed = false;
   if (status & kStatusTimeout) {
     set_error("a bounded device wait gave up");
     return MF_ETIMEOUT;

@@ -31,7 +31,7 @@ def mf():
 
 def _tight():
     p = W.paper_scale()
-    return W.set_scenario(p, 17, (-0.2, 0.3))
+    return W.set_scenario(p, 17, W.TIGHT_SLA)
 
 
 def _same(got, ref):
@@ -69,3 +69,40 @@ def test_noalloc_rejects_sizes_beyond_its_limits(mf):
     with pytest.raises(mf.MFError) as e:
         mf.search_exhaustive_noalloc(big, 8)
     assert e.value.status == mf.MF_EINVAL and "MF_NOALLOC_MAX_WEIGHT_BYTES" in str(e.value)
+
+
+def test_noalloc_allocates_nothing_after_the_first_call(mf):
+    """The first call on a device reserves the array (the runtime loads the module
+    that holds it); later calls must leave the device's free memory exactly as it
+    was.  For contrast, creating a context and searching with it does allocate."""
+    import torch
+    prob = W.paper_scale()
+    mf.search_exhaustive_noalloc(prob, 8)  # the first call on this device
+    torch.cuda.synchronize()
+    free0 = torch.cuda.mem_get_info()[0]
+    for k in (1, 8, 64):
+        mf.search_exhaustive_noalloc(prob, k)
+        mf.search_exhaustive_noalloc(W.tiny(), k, chunk=1 << 10)
+    torch.cuda.synchronize()
+    assert torch.cuda.mem_get_info()[0] == free0
+    with mf.Context(prob) as ctx:
+        ctx.search(8)
+        torch.cuda.synchronize()
+        assert torch.cuda.mem_get_info()[0] < free0
+
+
+def test_noalloc_matches_the_oracle(mf, oracle_mod):
+    """The same result as the CPU oracle's exhaustive search (fp64 on the same fp32
+    inputs), under the search contract of the other parity tests: the count within
+    the number of candidates near a threshold, every reported entry feasible and
+    scored within the fp32 tolerance, indices exact where scores are well separated,
+    on a problem whose SLA mask binds."""
+    from _parity import check_search, near_threshold
+    prob = _tight()
+    o = oracle_mod.Oracle(prob)
+    ti, ts, cnt = o.exhaustive(32)
+    _, _, pr, ag = o.score_list(np.arange(o.space_size(), dtype=np.uint64), with_pred=True)
+    bound = int(near_threshold(prob, pr, ag).sum())
+    assert 0 < cnt < o.space_size()
+    res = mf.search_exhaustive_noalloc(prob, 32)
+    check_search(o, prob, res, 32, (ti, ts), cnt, near_count_bound=bound)
