@@ -448,6 +448,19 @@ k_ga_persist(const Params P, const GaArgs g, const GaPersist G) {
   if (tid == 0) s_abort = 0;
   __syncthreads();
 
+  if (P.wait_test) {  // the timeout test: a record word that nothing writes, a few polls
+    if (tid == 0) {
+      bool got = false;
+      for (uint32_t n = 0; n < P.wait_test && !got; ++n)
+        got = has_tag(ld_word(&G.best[0].fw), 0xFFFFFFFFu);
+      if (!got) {
+        atomicOr(P.status, kStatusTimeout);
+        s_abort = 1;
+      }
+    }
+    __syncthreads();
+    if (s_abort) return;
+  }
   const uint64_t sd = *G.seed;
   const int c0 = blockIdx.x * SM;
   const int ns = min(SM, pop - c0);

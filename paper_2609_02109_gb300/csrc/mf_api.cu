@@ -576,6 +576,12 @@ mf_status mf_get_stats(const mf_ctx* ctx, mf_stats* out) {
   return MF_OK;
 }
 
+mf_status mf_debug_wait_test(mf_ctx* ctx, uint32_t polls) {
+  if (!ctx) return einval("ctx is NULL");
+  ctx->P.wait_test = polls;
+  return MF_OK;
+}
+
 mf_status mf_check_device_status(mf_ctx* ctx, void* stream) {
   if (!ctx) return einval("ctx is NULL");
   DeviceGuard guard(ctx->device);

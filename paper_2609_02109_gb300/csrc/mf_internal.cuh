@@ -38,6 +38,10 @@ struct Params {
   float u_omega[MF_MAX_MODELS], u_tau[MF_MAX_MODELS], u_cost[MF_MAX_MODELS];
   int32_t u_prev[MF_MAX_MODELS];
   float u_alpha, u_beta, u_delta;
+  // Test of the timeout path (mf_debug_wait_test): when non-zero, the kernels with
+  // bounded device waits first wait on a flag that nothing sets, giving up after this
+  // many polls, and then run to their end as after any wait that gave up.
+  uint32_t wait_test;
 };
 
 // Tensor-core path: operand images and the per-CTA layout (filled by tc_prepare).

@@ -25,7 +25,7 @@ _EXPORTS = ["mf_status_string", "mf_last_error", "mf_create", "mf_destroy", "mf_
             "mf_set_objective", "mf_score_batch", "mf_search_range", "mf_search_exhaustive",
             "mf_ga_generation", "mf_ga_init", "mf_ga_step", "mf_ga_run", "mf_check_device_status",
             "mf_get_stats", "mf_search_exhaustive_noalloc", "mf_fc_set", "mf_fc_table", "mf_fc_search",
-            "mf_vram_feasible", "mf_set_utility", "mf_fc_ga_run"]
+            "mf_vram_feasible", "mf_set_utility", "mf_fc_ga_run", "mf_debug_wait_test"]
 
 
 class MFError(RuntimeError):
@@ -94,6 +94,7 @@ def _load() -> C.CDLL:
     lib.mf_ga_step.argtypes = [vp, C.POINTER(_GAParams), u64, i32, vp, vp, vp, vp]
     lib.mf_ga_run.argtypes = [vp, C.POINTER(_GAParams), u64, vp, vp, vp]
     lib.mf_check_device_status.argtypes = [vp, vp]
+    lib.mf_debug_wait_test.argtypes = [vp, C.c_uint32]
     lib.mf_get_stats.argtypes = [vp, C.POINTER(_Stats)]
     lib.mf_search_exhaustive_noalloc.argtypes = [C.POINTER(_Problem), i32, u64, C.POINTER(_Result), vp]
     lib.mf_fc_set.argtypes = [vp, C.POINTER(_FcParams), vp]
@@ -367,3 +368,8 @@ class Context:
     def check_status(self) -> int:
         """MF_OK, or the status of the first device-reported problem (clears it)."""
         return int(_lib.mf_check_device_status(self._h, _stream(self.device)))
+
+    def debug_wait_test(self, polls: int) -> None:
+        """mf_debug_wait_test: with polls > 0 the context's waiting kernels first wait on
+        a flag that nothing sets and give up (tests of the timeout path); 0 restores."""
+        _check(_lib.mf_debug_wait_test(self._h, int(polls)), "mf_debug_wait_test")
