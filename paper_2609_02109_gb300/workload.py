@@ -25,7 +25,10 @@ in for the profiled LLM/YOLO landscape, which is not available:
 * predictor weights: Xavier/Glorot uniform U(+-sqrt(6 / (fan_in + fan_out)));
   biases ~ U(+-1 / sqrt(fan_in)); one distinct MLP per model;
 * SLA latency ceilings ~ U(0.5, 2.0); objective weights ~ U(0.5, 1.5);
-* the "tight" variant draws SLA ~ U(-0.2, 0.3) so that the latency mask binds.
+* the "tight" variant draws SLA ~ U(0.1, 0.9) (TIGHT_SLA) so that the latency mask binds
+  on part of the space (the synthetic predictors' latencies are of order 0-0.7; which
+  scenario seeds leave a feasible fraction strictly between 0 and 1 is checked by the
+  tests that use them).
 
 Predictor weights of model i are packed, PyTorch ``Linear`` convention
 (weight[out][in]), as W1[h1][d_in], b1[h1], (W2[h2][h1], b2[h2] if h2 > 0),
@@ -145,6 +148,10 @@ def make_problem(n_options, d_local, h1, h2, seed, vram_cap, objective="weighted
     return prob
 
 
+# SLA ceilings under which the latency mask binds on part of a space.
+TIGHT_SLA = (0.1, 0.9)
+
+
 def set_scenario(prob: dict, scenario_seed: int, sla_range=(0.5, 2.0)) -> dict:
     """Redraw the SLA ceilings and objective weights (the per-scenario inputs)."""
     n = int(prob["n_options"].size)
@@ -187,7 +194,7 @@ def _ints(seed: int, purpose: int, model: int, n: int, lo: int, hi: int) -> np.n
 
 
 def integer_landscape(n_options, seed: int, vram_cap: float, objective="weighted_thr",
-                      soft_penalty=0.0) -> dict:
+                      soft_penalty=0.0, coupled: bool = False) -> dict:
     """A d_L = 8, 12->64->64->2 problem whose every input is a small integer.
 
     Local features in [-2, 2], demands in [1, 9] (three columns), W1 in [-1, 1]
@@ -197,6 +204,10 @@ def integer_landscape(n_options, seed: int, vram_cap: float, objective="weighted
     below 2**24 in magnitude, so fp32 and fp64 evaluation in any summation order
     give the same number and a GA run is reproducible bit for bit across
     implementations.
+
+    coupled: keep W1's four aggregate columns (integers in [-1, 1]) and feed the
+    aggregate unscaled (agg_scale = 1), so each predictor sees the candidate's
+    summed demands and N; the values stay integers (below 2**24 for N <= 5).
     """
     n_options = np.asarray(n_options, dtype=np.int32)
     n = int(n_options.size)
@@ -208,7 +219,8 @@ def integer_landscape(n_options, seed: int, vram_cap: float, objective="weighted
         dems.append(np.stack([_ints(seed, P_SM, i, k, 1, 9), _ints(seed, P_VRAM, i, k, 1, 9),
                               _ints(seed, P_BW, i, k, 1, 9)], axis=1))
         w1 = _ints(seed, P_W1, i, h * d_in, -1, 1).reshape(h, d_in)
-        w1[:, d:] = 0.0
+        if not coupled:
+            w1[:, d:] = 0.0
         ws.append(np.concatenate([w1.ravel(), _ints(seed, P_B1, i, h, -2, 2),
                                   _ints(seed, P_W2, i, h * h, -1, 1), _ints(seed, P_B2, i, h, -2, 2),
                                   _ints(seed, P_W3, i, 2 * h, -1, 1), _ints(seed, P_B3, i, 2, -2, 2)]))
@@ -217,9 +229,9 @@ def integer_landscape(n_options, seed: int, vram_cap: float, objective="weighted
         local_feats=np.ascontiguousarray(np.concatenate(locs, axis=0), dtype=np.float32),
         demand=np.ascontiguousarray(np.concatenate(dems, axis=0), dtype=np.float32),
         weights=np.ascontiguousarray(np.concatenate(ws), dtype=np.float32),
-        agg_scale=default_agg_scale(n), vram_cap=float(vram_cap),
+        agg_scale=np.ones(4, dtype=np.float32) if coupled else default_agg_scale(n), vram_cap=float(vram_cap),
         soft_penalty=float(soft_penalty), objective=objective, out_act="identity", precision="fp32",
-        sla=_ints(seed, P_SLA, 0, n, 40, 120), obj_w=_ints(seed, P_OBJW, 0, n, 1, 3),
+        sla=_ints(seed, P_SLA, 0, n, 40, 120) * (4 if coupled else 1), obj_w=_ints(seed, P_OBJW, 0, n, 1, 3),
         scenario_seed=int(seed),
     )
 

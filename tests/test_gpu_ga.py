@@ -49,6 +49,10 @@ CASES = {
     "one_model": ([200], 8, 9.0, "weighted_thr", dict(W.GA_PARAMS, pop=50, gens=25, mutation_p=0.2)),
     "pop_two_one_gen": ([6, 7, 8], 9, 20.0, "weighted_thr", dict(W.GA_PARAMS, pop=2, gens=1)),
     "single_generation": ([12, 9, 9, 9, 9], 5, 30.0, "weighted_thr", dict(W.GA_PARAMS, gens=1)),
+    # the predictors see the candidate's own aggregate (W1's aggregate columns in use,
+    # unscaled): the cooperative kernel's coupled fitness, not only its winner
+    "coupled_paper_shape": ([12, 9, 9, 9, 9], 5, 30.0, "weighted_thr", dict(W.GA_PARAMS), True),
+    "coupled_four_models": ([16] * 4, 6, 25.0, "soft_lat", dict(W.GA_PARAMS, pop=100, gens=60), True),
     # eight models take a whole SM per CTA: a population above 8 per SM cannot be resident
     "graph_fallback_pop_over_8_per_sm": ([5] * 8, 7, 45.0, "weighted_thr",
                                          dict(W.GA_PARAMS, pop=9 * 160, gens=12)),
@@ -56,9 +60,10 @@ CASES = {
 
 
 def _problem(name):
-    opts, seed, cap, objective, _ = CASES[name]
+    opts, seed, cap, objective = CASES[name][:4]
+    coupled = len(CASES[name]) > 5 and CASES[name][5]
     return W.integer_landscape(opts, seed, cap, objective=objective,
-                               soft_penalty=0.5 if objective == "soft_lat" else 0.0)
+                               soft_penalty=0.5 if objective == "soft_lat" else 0.0, coupled=coupled)
 
 
 @pytest.mark.parametrize("name", list(CASES))

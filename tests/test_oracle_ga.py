@@ -140,23 +140,29 @@ def test_ga_finds_optimum_of_tiny_space(oracle_mod):
     assert list(genome) == list(o.decode(int(ti[0])))
 
 
-@pytest.mark.parametrize("opts,seed,cap", [([12, 9, 9, 9, 9], 5, 30.0), ([5] * 8, 7, 45.0)])
-def test_integer_landscape_is_exact_in_any_order(oracle_mod, opts, seed, cap):
+@pytest.mark.parametrize("opts,seed,cap,coupled", [([12, 9, 9, 9, 9], 5, 30.0, False), ([5] * 8, 7, 45.0, False),
+                                                  ([12, 9, 9, 9, 9], 5, 30.0, True), ([16] * 4, 6, 25.0, True)])
+def test_integer_landscape_is_exact_in_any_order(oracle_mod, opts, seed, cap, coupled):
     """The premise of the bit-exact GA tests on the GPU: in the integer landscapes
     every input is an integer and the largest value any partial sum can reach is
-    below 2**24, so fp32 arithmetic is exact whatever the summation order."""
-    prob = W.integer_landscape(opts, seed, cap, objective="soft_lat", soft_penalty=0.5)
+    below 2**24, so fp32 arithmetic is exact whatever the summation order.  In the
+    coupled variant the predictors also see the unscaled aggregate (summed demands
+    and N), which stays an integer."""
+    prob = W.integer_landscape(opts, seed, cap, objective="soft_lat", soft_penalty=0.5, coupled=coupled)
     n, d, h = len(opts), 8, 64
     per = W.param_count(d, h, h)
-    for a in (prob["local_feats"], prob["demand"], prob["weights"], prob["sla"], prob["obj_w"]):
+    for a in (prob["local_feats"], prob["demand"], prob["weights"], prob["sla"], prob["obj_w"]) + \
+            ((prob["agg_scale"],) if coupled else ()):
         assert np.all(a == np.round(a))
     w = prob["weights"].reshape(n, per).astype(np.float64)
     x = float(np.abs(prob["local_feats"]).max())
+    agg = np.append(n * np.abs(prob["demand"]).max(axis=0), n) * (prob["agg_scale"] if coupled else 0.0)
     b1 = h * (d + 4)
     for i in range(n):
         W1 = w[i, :b1].reshape(h, d + 4)
-        assert np.all(W1[:, d:] == 0)  # the aggregate inputs do not enter
-        h1 = d * x * np.abs(W1).max() + np.abs(w[i, b1:b1 + h]).max()
+        assert np.any(W1[:, d:] != 0) if coupled else np.all(W1[:, d:] == 0)
+        h1 = d * x * np.abs(W1[:, :d]).max() + float(np.abs(W1[:, d:]).max(axis=0) @ agg) + \
+            np.abs(w[i, b1:b1 + h]).max()
         o2 = b1 + h
         h2 = h * h1 * np.abs(w[i, o2:o2 + h * h]).max() + np.abs(w[i, o2 + h * h:o2 + h * h + h]).max()
         o3 = o2 + h * h + h
