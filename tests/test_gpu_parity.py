@@ -38,12 +38,12 @@ def _score_all(ctx, idx_np, with_pred=True):
 
 def _problems():
     tight = W.paper_scale()
-    W.set_scenario(tight, 17, (-0.2, 0.3))
+    W.set_scenario(tight, 17, W.TIGHT_SLA)
     sig = W.random_small(21, n_models=4, max_options=8, h2=32, vram_cap=40.0, out_act="sigmoid",
-                         sla_range=(0.3, 0.7))
+                         sla_range=(0.4, 0.9))
     soft = W.make_problem([3] * 8, 16, 128, 128, 4, 180.0, objective="soft_lat", soft_penalty=0.1,
                           sla_range=(-0.2, 0.3))
-    odd = W.make_problem([5, 7, 3], 3, 20, 10, 8, 30.0, sla_range=(-0.1, 0.3))
+    odd = W.make_problem([5, 7, 3], 3, 20, 10, 8, 30.0, sla_range=W.TIGHT_SLA)
     return {"hand": W.hand_example(), "tiny": W.tiny(), "paper": W.paper_scale(), "tight": tight,
             "sigmoid": sig, "soft8": soft, "odd_shape": odd}
 
@@ -153,7 +153,7 @@ def test_out_of_range_index_raises_device_status(mf):
 def test_set_objective_changes_scores(mf, oracle_mod):
     prob = W.paper_scale()
     with mf.Context(prob) as ctx:
-        W.set_scenario(prob, 123, (-0.2, 0.3))
+        W.set_scenario(prob, 123, (-0.1, 0.8))
         ctx.set_objective(prob["sla"], prob["obj_w"])
         res = ctx.search(8)
     o = oracle_mod.Oracle(prob)

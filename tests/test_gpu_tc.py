@@ -28,19 +28,19 @@ def mf():
 def _problems():
     paper = W.paper_scale(precision="bf16")
     tight = W.paper_scale(precision="bf16")
-    W.set_scenario(tight, 17, (-0.2, 0.3))
+    W.set_scenario(tight, 17, W.TIGHT_SLA)
     # the stress per-model shape (d_L 16 -> K1 = 32, 128-wide layers, soft latency)
     # on three models, so all weights fit shared memory
     stress3 = W.make_problem([16] * 3, 16, 128, 128, 4, 180.0, objective="soft_lat",
                              soft_penalty=0.1, precision="bf16", sla_range=(-0.2, 0.3))
     # odd d_L (padded), one hidden layer, sigmoid outputs, binding VRAM cap
     odd = W.make_problem([7, 9, 6], 7, 32, 0, 12, 30.0, out_act="sigmoid", precision="bf16",
-                         sla_range=(0.3, 0.7))
+                         sla_range=(0.4, 0.9))
     # paper's 64-32 predictor shape, eight models (16 D3 columns)
-    p6432 = W.make_problem([4] * 8, 8, 64, 32, 13, 100.0, precision="bf16", sla_range=(-0.1, 0.4))
+    p6432 = W.make_problem([4] * 8, 8, 64, 32, 13, 100.0, precision="bf16", sla_range=W.TIGHT_SLA)
     # five 20->128->128->2 models: 240 KB of bf16 weights, staged in two passes (3 + 2 models)
     multipass = W.make_problem([3, 4, 2, 3, 2], 16, 128, 128, 5, 180.0, precision="bf16",
-                               sla_range=(-0.2, 0.3))
+                               sla_range=(0.2, 0.8))
     return {"paper": paper, "tight": tight, "stress3": stress3, "odd": odd, "p6432": p6432,
             "multipass": multipass}
 

@@ -190,7 +190,7 @@ def _separable(prob):
     return prob
 
 
-@pytest.mark.parametrize("sla_range", [(0.5, 2.0), (-0.2, 0.3)])
+@pytest.mark.parametrize("sla_range", [(0.5, 2.0), W.TIGHT_SLA])
 def test_separable_closed_form(oracle_mod, sla_range):
     """Separable case: argmax = per-model argmax of w_i thr_i over the options
     meeting SLA_i; feasible count = prod_i #{o : lat_i(o) <= SLA_i}."""
@@ -279,7 +279,7 @@ def _brute_topk(o, k):
 @pytest.mark.parametrize("seed", [1, 2, 3, 4, 5])
 def test_exhaustive_equals_brute_force(oracle_mod, seed):
     prob = W.random_small(seed, n_models=4, max_options=7, h2=16, vram_cap=35.0,
-                          sla_range=(-0.2, 0.3))
+                          sla_range=(0.3, 1.0))
     o = _O(oracle_mod, prob)
     k = 10
     keep, s, cnt = _brute_topk(o, k)
@@ -302,7 +302,7 @@ def test_ties_ordered_by_index(oracle_mod):
 
 def test_candidate_order_invariance(oracle_mod):
     prob = W.paper_scale()
-    W.set_scenario(prob, 5, (-0.2, 0.3))
+    W.set_scenario(prob, 5, (0.4, 0.9))
     o = _O(oracle_mod, prob)
     rs = np.random.default_rng(3)
     idx = rs.integers(0, o.space_size(), size=500).astype(np.uint64)
@@ -365,3 +365,31 @@ def test_pred_scale_hand_value(oracle_mod):
     J, f, pred, _ = o.score_digits([0])
     assert pred[0, 0] == pytest.approx(0.25)
     np.testing.assert_allclose(o.pred_scale(np.array([0], np.uint64))[0, 0], [0.75, 0.0], atol=1e-12)
+
+
+def _feasible_fraction(oracle_mod, prob, sample=40000):
+    o = _O(oracle_mod, prob)
+    n = o.space_size()
+    idx = np.arange(n, dtype=np.uint64) if n <= sample else \
+        np.random.default_rng(0).integers(0, n, sample).astype(np.uint64)
+    return float(o.score_list(idx)[1].mean())
+
+
+def test_scenarios_that_exercise_the_masks_bind_on_part_of_the_space(oracle_mod):
+    """The parity tests' and the benchmark's mask scenarios leave a feasible fraction
+    strictly between 0 and 1: a mask that rejects everything (or nothing) would let a
+    wrong feasibility test pass unnoticed."""
+    import test_gpu_parity as tp
+    import test_gpu_tc as tt
+    cases = {"parity." + k: tp.PROBLEMS[k] for k in ("tight", "odd_shape", "sigmoid")}
+    cases.update({"tc." + k: tt.PROBLEMS[k] for k in ("tight", "odd", "p6432", "multipass")})
+    for seed in (1, 2, 3, 4, 5):
+        cases[f"brute{seed}"] = W.random_small(seed, n_models=4, max_options=7, h2=16, vram_cap=35.0,
+                                               sla_range=(0.3, 1.0))
+    cases["order"] = W.set_scenario(W.paper_scale(), 5, (0.4, 0.9))
+    cases["set_objective"] = W.set_scenario(W.paper_scale(), 123, (-0.1, 0.8))
+    large = W.large(precision="fp32")
+    cases["bench_tight"] = W.set_scenario(large, 31, W.TIGHT_SLA)
+    for name, prob in cases.items():
+        fr = _feasible_fraction(oracle_mod, prob)
+        assert 0.0 < fr < 1.0, (name, fr)

@@ -47,7 +47,7 @@ def _rank_main(rank, world, port, k, name, out_dir):
     os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
     dist.init_process_group("gloo", rank=rank, world_size=world)
     from oracle import oracle
-    prob = {"tight": W.set_scenario(W.paper_scale(), 17, (-0.2, 0.3)), "tiny": W.tiny()}[name]
+    prob = {"tight": W.set_scenario(W.paper_scale(), 17, W.TIGHT_SLA), "tiny": W.tiny()}[name]
     o = oracle.Oracle(prob)
     lo, hi = shard.shard_range(o.space_size(), rank, world)
     ti, ts, cnt = o.exhaustive(k, lo=lo, hi=hi)
@@ -64,10 +64,53 @@ def test_gloo_ranks_merge_to_the_single_range_result(oracle_mod, tmp_path, world
     import torch.multiprocessing as mp
     mp.start_processes(_rank_main, args=(world, _free_port(), k, name, str(tmp_path)), nprocs=world,
                        join=True, start_method="spawn")
-    prob = {"tight": W.set_scenario(W.paper_scale(), 17, (-0.2, 0.3)), "tiny": W.tiny()}[name]
+    prob = {"tight": W.set_scenario(W.paper_scale(), 17, W.TIGHT_SLA), "tiny": W.tiny()}[name]
     ti, ts, cnt = oracle_mod.Oracle(prob).exhaustive(k)
     for r in range(world):
         got = np.load(tmp_path / f"r{r}.npz")
         assert int(got["count"]) == cnt
+        assert np.array_equal(got["idx"], np.asarray(ti, np.uint64))
+        assert np.array_equal(got["score"], np.asarray(ts, np.float32))
+
+
+class _OracleContext:
+    """The two members of the binding's Context that search_sharded uses (space_size,
+    search over an index range), served by the oracle: a rank's GPU on the CPU."""
+
+    def __init__(self, prob):
+        from oracle import oracle
+        self.o = oracle.Oracle(prob)
+        self.space_size = self.o.space_size()
+
+    def search(self, k, lo=0, hi=None, chunk=0):
+        ti, ts, cnt = self.o.exhaustive(k, lo=lo, hi=hi)
+        return dict(best_idx=int(ti[0]), best_score=float(ts[0]), count=cnt,
+                    topk_idx=np.asarray(ti, np.uint64), topk_score=np.asarray(ts, np.float32))
+
+
+def _sharded_main(rank, world, port, k, out_dir):
+    import torch.distributed as dist
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    prob = W.set_scenario(W.paper_scale(), 17, W.TIGHT_SLA)
+    merged = shard.search_sharded(_OracleContext(prob), k)
+    np.savez(os.path.join(out_dir, f"s{rank}.npz"), idx=merged["topk_idx"], score=merged["topk_score"],
+             count=merged["count"], best=merged["best_idx"])
+    dist.barrier()
+    dist.destroy_process_group()
+
+
+def test_search_sharded_end_to_end_on_gloo_ranks(oracle_mod, tmp_path):
+    """The multi-GPU step of the benchmark (shard.search_sharded: this rank's range,
+    then the all-gather and merge) on two CPU ranks equals the single search."""
+    import torch.multiprocessing as mp
+    world, k = 2, 32
+    mp.start_processes(_sharded_main, args=(world, _free_port(), k, str(tmp_path)), nprocs=world,
+                       join=True, start_method="spawn")
+    prob = W.set_scenario(W.paper_scale(), 17, W.TIGHT_SLA)
+    ti, ts, cnt = oracle_mod.Oracle(prob).exhaustive(k)
+    for r in range(world):
+        got = np.load(tmp_path / f"s{r}.npz")
+        assert int(got["count"]) == cnt and int(got["best"]) == int(ti[0])
         assert np.array_equal(got["idx"], np.asarray(ti, np.uint64))
         assert np.array_equal(got["score"], np.asarray(ts, np.float32))
