@@ -13,8 +13,11 @@ reported in the same JSON line.
     python bench.py [--gpus N] [--steps K] [--warmup W] [--precision bf16|fp32]
     python bench.py --impl reference ...   # the CPU oracle as the reference arm
 
-Multi-GPU (torchrun, one rank per GPU): every rank searches its own scenario
-(independent problems, no collective in the data path): weak scaling.
+Multi-GPU (torchrun, one rank per GPU): the ranks split the same space into
+contiguous index ranges, search their range on their GPU and exchange the k best
+(score, index) pairs and the feasible counts in one NCCL all-gather
+(paper_2609_02109_gb300.shard.search_sharded): the total work per step is fixed,
+so the scaling is strong.
 """
 from __future__ import annotations
 
@@ -41,9 +44,9 @@ K_TOP = 32
 CHUNK = 1 << 24
 L2_FLUSH_BYTES = 256 << 20
 
-# DRAM bytes (read + write) of one scoring launch from the ncu capture summarised in
-# profiles/k_score_tc_large_n6.md, valid only while the kernel's sources are the ones
-# that were captured (sha256 prefix of k_tc.cu + mf_internal.cuh)
+# DRAM bytes (read + write) of one scoring launch from the ncu capture of the scoring
+# kernel on this workload, valid only while the kernel's sources are the ones that were
+# captured (sha256 prefix of k_tc.cu + mf_internal.cuh)
 NCU_TRAFFIC = {"bf16": ("739c026bcbb59df6", 2116864)}
 
 
@@ -213,6 +216,93 @@ def run_reference(args):
 # ---------------------------------------------------------------------------
 # GPU arm
 # ---------------------------------------------------------------------------
+def fp32_peak(torch, device):
+    """The fp32 FMA rate of a cuBLAS fp32 GEMM with TF32 off (8192^3, best of five
+    after two warm-ups): the measured stand-in for the FP32 pipe's peak, as the bf16
+    peak is cuBLAS's bf16 GEMM."""
+    prev = torch.backends.cuda.matmul.allow_tf32
+    torch.backends.cuda.matmul.allow_tf32 = False
+    try:
+        n = 8192
+        a = torch.randn(n, n, device=f"cuda:{device}", dtype=torch.float32)
+        b = torch.randn(n, n, device=f"cuda:{device}", dtype=torch.float32)
+        for _ in range(2):
+            torch.matmul(a, b)
+        best = float("inf")
+        stream = torch.cuda.current_stream(device)
+        for _ in range(5):
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            torch.matmul(a, b)
+            e1.record(stream)
+            e1.synchronize()
+            best = min(best, e0.elapsed_time(e1))
+        del a, b
+        return 2.0 * n ** 3 / (best / 1e3) / 1e12
+    finally:
+        torch.backends.cuda.matmul.allow_tf32 = prev
+
+
+def tight_throughput(mf, torch, device):
+    """The large workload's space with SLA ceilings ~ U(0.1, 0.9), where the latency
+    mask binds: the SLA mask, the bf16 shortlist band around the ceilings and the fp32
+    re-scoring of the shortlist are all on the timed path."""
+    prob = W.large(precision="bf16")
+    W.set_scenario(prob, 31, W.TIGHT_SLA)
+    n = 24 ** 6
+    stream = torch.cuda.current_stream(device)
+    peaks, src = _peaks()
+    with mf.Context(prob, device=device) as ctx:
+        ctx.search(K_TOP, chunk=CHUNK)
+        ms, score_ms = [], []
+        for _ in range(3):
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            torch.cuda.synchronize(device)
+            e0.record(stream)
+            res = ctx.search(K_TOP, chunk=CHUNK)
+            e1.record(stream)
+            e1.synchronize()
+            st = ctx.stats()
+            ms.append(e0.elapsed_time(e1))
+            score_ms.append(st["score_ms_last"] / st["score_launches_last"])
+    launch_ms = float(np.median(score_ms))
+    achieved = flops_per_candidate(prob) * (n / 12) / (launch_ms / 1e3) / 1e12
+    peak = float(peaks["bf16_tflops"])
+    return {"workload": "large space (N=6 x 24 options), scenario 31 with SLA ~ U(0.1, 0.9): latency mask binds",
+            "value": n / (float(np.median(ms)) / 1e3), "unit": UNIT, "ms": float(np.median(ms)),
+            "feasible_fraction": res["count"] / n, "count": res["count"], "best": res["best_idx"],
+            "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                         "frac": achieved / peak, "launch_ms": launch_ms,
+                         "peak_source": f"{src} bf16 burst"}}
+
+
+def exact_throughput(mf, torch, device, sgemm_tflops):
+    """The exact fp32 search (CUDA-core scorer) of the large workload."""
+    prob = W.large(precision="fp32")
+    n = 24 ** 6
+    stream = torch.cuda.current_stream(device)
+    with mf.Context(prob, device=device) as ctx:
+        ctx.search(K_TOP, chunk=CHUNK)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize(device)
+        e0.record(stream)
+        res = ctx.search(K_TOP, chunk=CHUNK)
+        e1.record(stream)
+        e1.synchronize()
+        st = ctx.stats()
+    ms = e0.elapsed_time(e1)
+    launch_ms = st["score_ms_last"] / st["score_launches_last"]
+    achieved = flops_per_candidate(prob) * (n / st["score_launches_last"]) / (launch_ms / 1e3) / 1e12
+    return {"workload": "large exhaustive, exact fp32 path", "value": n / (ms / 1e3), "unit": UNIT, "ms": ms,
+            "best": res["best_idx"], "count": res["count"],
+            "roofline": {"bound": "fp32", "achieved": achieved, "peak": sgemm_tflops, "unit": "TFLOP/s",
+                         "frac": achieved / sgemm_tflops, "launch_ms": launch_ms,
+                         "peak_source": "measured cuBLAS fp32 GEMM (TF32 off), this run"}}
+
+
 def stress_throughput(mf, torch, device):
     """The stress workload (2^32 candidates, bf16, eight 20->128->128->2 predictors in
     three shared-memory passes), one warm-up and one timed search."""
@@ -377,17 +467,22 @@ def run_gpu(args):
         dist.barrier()
     from paper_2609_02109_gb300 import mf
 
+    from paper_2609_02109_gb300 import shard
+
     prec = args.precision
-    prob = W.large(precision=prec)
-    if rank:
-        W.set_scenario(prob, 3 + 1000 * rank)
+    prob = W.large(precision=prec)  # every rank: the same space, its own index range
     n_cand = 24 ** 6
     device = local
     stream = torch.cuda.current_stream(device)
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=f"cuda:{device}")
+    def step(ctx):
+        if dist:  # this rank's range, then the all-gather of the k best pairs and the counts
+            return shard.search_sharded(ctx, K_TOP, chunk=CHUNK, device=torch.device("cuda", device))
+        return ctx.search(K_TOP, chunk=CHUNK)
+
     with mf.Context(prob, device=device) as ctx:
         for _ in range(args.warmup):
-            ctx.search(K_TOP, chunk=CHUNK)
+            step(ctx)
         step_ms, score_ms, launches, score_launches = [], [], 0, 0
         res = None
         with ClockSampler(device) as clk:
@@ -399,7 +494,7 @@ def run_gpu(args):
                 e0 = torch.cuda.Event(enable_timing=True)
                 e1 = torch.cuda.Event(enable_timing=True)
                 e0.record(stream)
-                res = ctx.search(K_TOP, chunk=CHUNK)
+                res = step(ctx)
                 e1.record(stream)
                 e1.synchronize()
                 step_ms.append(e0.elapsed_time(e1))
@@ -415,26 +510,27 @@ def run_gpu(args):
             t = torch.tensor([total_ms], device=f"cuda:{device}")
             dist.all_reduce(t, op=dist.ReduceOp.MAX)
             total_ms = float(t.item())
-        value = world * n_cand * args.steps / (total_ms / 1e3)
+        value = n_cand * args.steps / (total_ms / 1e3)  # the whole space per step, over all ranks
         feasible_frac = res["count"] / n_cand
 
         # roofline of the scoring kernel: algorithmic FLOPs per launch / mean launch time
         fpc = flops_per_candidate(prob)
         per_launch_ms = float(sum(score_ms)) / max(score_launches, 1)
-        per_launch_flops = fpc * n_cand / (score_launches / args.steps)
+        lo, hi = shard.shard_range(n_cand, rank, world)
+        per_launch_flops = fpc * (hi - lo) / (score_launches / args.steps)
         peaks, src = _peaks()
         achieved = per_launch_flops / (per_launch_ms / 1e3) / 1e12
+        sgemm = fp32_peak(torch, device) if (rank == 0 and (prec == "fp32" or not args.no_stress)) else None
         if prec == "bf16":
-            peak = float(peaks["bf16_tflops_sustained"])
+            # launches of about a millisecond inside a step of tens: the burst peak applies
+            peak = float(peaks["bf16_tflops"])
             roof = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                    "frac": achieved / peak, "frac_burst": achieved / float(peaks["bf16_tflops"]),
-                    "peak_source": f"{src} bf16 sustained (burst {peaks['bf16_tflops']})"}
+                    "frac": achieved / peak, "frac_sustained": achieved / float(peaks["bf16_tflops_sustained"]),
+                    "peak_source": f"{src} bf16 burst (sustained {peaks['bf16_tflops_sustained']})"}
         else:
-            sms = torch.cuda.get_device_properties(device).multi_processor_count
-            peak = sms * 128 * 2 * float(peaks.get("sm_max_mhz", 2070.0)) * 1e6 / 1e12
-            roof = {"bound": "alu", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                    "frac": achieved / peak,
-                    "peak_source": f"{sms} SMs x 128 FP32 lanes x 2 FLOP x {peaks.get('sm_max_mhz', 2070.0)} MHz"}
+            roof = {"bound": "fp32", "achieved": achieved, "peak": sgemm, "unit": "TFLOP/s",
+                    "frac": achieved / sgemm if sgemm else None,
+                    "peak_source": "measured cuBLAS fp32 GEMM (TF32 off), this run"}
         roof.update({"traffic": _traffic(prec), "kernel": "scoring kernel (one launch per 2^24 candidates)",
                      "flops_per_candidate": fpc, "launch_ms": per_launch_ms})
 
@@ -444,15 +540,23 @@ def run_gpu(args):
             torch.cuda.synchronize(device)
             t0 = time.perf_counter()
             with mf.Context(prob, device=device) as c2:
-                c2.search(K_TOP, chunk=CHUNK)
+                step(c2)
                 st2 = c2.stats()
             e2e_ms.append(1e3 * (time.perf_counter() - t0))
-        e2e = {"value": n_cand / (statistics.median(e2e_ms) / 1e3), "unit": UNIT,
+        e2e_med = statistics.median(e2e_ms)
+        if dist:
+            t = torch.tensor([e2e_med], device=f"cuda:{device}")
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e2e_med = float(t.item())
+        e2e = {"value": n_cand / (e2e_med / 1e3), "unit": UNIT,
                "h2d_bytes_per_step": int(st2["h2d_bytes_create"]),
                "d2h_bytes_per_step": int(st2["d2h_bytes_last"]),
                "how": "mf_create from host arrays + mf_search_exhaustive + mf_destroy, host wall clock, median"}
 
     stress = stress_throughput(mf, torch, device) if rank == 0 and not args.no_stress else None
+    tight = tight_throughput(mf, torch, device) if rank == 0 and not args.no_stress else None
+    exact = exact_throughput(mf, torch, device, sgemm) if rank == 0 and not args.no_stress and prec == "bf16" \
+        else None
     fixed = fixed_context_throughput(mf, torch, device) if rank == 0 and not args.no_stress else None
     ga = ga_latency(mf, torch, device, args.ga_decisions) if rank == 0 else None
     paper_ga = paper_ga_latency(mf, torch, device, args.ga_decisions) if rank == 0 else None
@@ -460,12 +564,17 @@ def run_gpu(args):
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
                 "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
-                "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if prec == "bf16" else "f32",
-                "data": "synthetic", "config": workload_config(prec), "roofline": roof,
+                "scaling": "strong", "vs_baseline": None, "dtype": "bf16" if prec == "bf16" else "f32",
+                "data": "synthetic", "config": dict(workload_config(prec), parallelism=(
+                    f"index-range split over {world} GPUs + all-gather of the k best" if world > 1 else "1 GPU")),
+                "roofline": roof,
                 "cpu_baseline": base, "e2e": e2e, "gpu_launches": launches, "clocks": clk.summary(),
                 "feasible_fraction": feasible_frac, "best": {"idx": res["best_idx"], "J": res["best_score"],
                                                              "count": res["count"]},
-                "ga": ga, "paper_ga": paper_ga, "stress": stress, "fixed_context": fixed}
+                "ga": ga, "paper_ga": paper_ga, "stress": stress, "fixed_context": fixed,
+                "tight": tight, "exact_fp32": exact,
+                "peaks": {"fp32_sgemm_tflops": sgemm, "fp32_sgemm_how": "cuBLAS fp32 GEMM 8192^3, TF32 off, "
+                          "best of 5 (the fp32 CUDA-core roofline)"} if sgemm else None}
         print(json.dumps(line), flush=True)
     if dist:
         dist.barrier()
