@@ -195,7 +195,8 @@ struct NamedSync128 {
 // The pipeline's top-k merge, out of line: it runs rarely and its registers stay off
 // the hot loop.
 __device__ __noinline__ void tc_topk_merge(const CtaTopK& tk, int row, int barid) {
-  topk_merge(tk, row, 128, NamedSync128{barid});
+  if (*tk.qn <= 128) topk_merge(tk, row, 128, NamedSync128{barid});
+  else topk_merge_sorted(tk, row, 128, NamedSync128{barid});
 }
 
 // The rest of a bounded wait, out of line: on giving up it flags the status word and
@@ -405,13 +406,13 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   auto topk = [&]() {
     CtaTopK tk;
     unsigned char* q = smem + T.sm_topk +
-                       (size_t)pipe * ((sizeof(uint64_t) + sizeof(float)) * (2 * (size_t)kcap + 128) + 16);
+                       (size_t)pipe * ((sizeof(uint64_t) + sizeof(float)) * (2 * (size_t)kcap + T.qcap) + 16);
     tk.li = reinterpret_cast<uint64_t*>(q); q += sizeof(uint64_t) * kcap;
     tk.ni = reinterpret_cast<uint64_t*>(q); q += sizeof(uint64_t) * kcap;
-    tk.qi = reinterpret_cast<uint64_t*>(q); q += sizeof(uint64_t) * 128;
+    tk.qi = reinterpret_cast<uint64_t*>(q); q += sizeof(uint64_t) * T.qcap;
     tk.ls = reinterpret_cast<float*>(q); q += sizeof(float) * kcap;
     tk.ns = reinterpret_cast<float*>(q); q += sizeof(float) * kcap;
-    tk.qs = reinterpret_cast<float*>(q); q += sizeof(float) * 128;
+    tk.qs = reinterpret_cast<float*>(q); q += sizeof(float) * T.qcap;
     tk.qn = reinterpret_cast<int*>(q);
     tk.k = kcap;
     return tk;
@@ -687,7 +688,10 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
         tk.qs[pos] = J;
         tk.qi[pos] = idx;
       }
-      if (named_bar_or(barid, 128, push)) tc_topk_merge(tk, row, barid);
+      // Candidates wait in the queue (against the list's k-th entry of the last merge)
+      // until another tile's 128 might not fit; then one merge takes them all.
+      named_bar(barid, 128);
+      if (*(volatile int*)tk.qn > T.qcap - 128) tc_topk_merge(tk, row, barid);
     }
   };
   auto load_d3 = [&](uint32_t (&d3)[D3W]) {
@@ -782,6 +786,11 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     load_d3(d3);
     finish_tile(d3, tile - gstride, digits + (buf ^ 1) * (MF_MAX_MODELS * 128));
   }
+  if (MODE == kTcRange && (!MP || T.pass_last)) {  // what is still queued joins the list
+    const CtaTopK tk = topk();
+    named_bar(barid, 128);
+    if (*(volatile int*)tk.qn > 0) tc_topk_merge(tk, row, barid);
+  }
 
   if (MODE == kTcRange && (!MP || T.pass_last)) {
     const CtaTopK tk = topk();
@@ -838,13 +847,17 @@ size_t umma_off(int r, int k, int kdim) {
 
 int round_up(int v, int a) { return (v + a - 1) / a * a; }
 
-size_t topk_bytes_pipe(int kcap) { return (sizeof(uint64_t) + sizeof(float)) * (2 * (size_t)kcap + 128) + 16; }
+size_t topk_bytes_pipe(int kcap, int qcap) {
+  return (sizeof(uint64_t) + sizeof(float)) * (2 * (size_t)kcap + qcap) + 16;
+}
 
 size_t image_bytes(const Params& P, int k1, int n3) {
   const int hl = P.h2 > 0 ? P.h2 : P.h1;
   const size_t per = (size_t)P.h1 * k1 * 2 + (size_t)P.h2 * (P.h1 + 16) * 2 + (size_t)n3 * hl * 2;
   return per * P.n_models;
 }
+
+constexpr uint32_t kSmemLimit = 227 * 1024 - 1024;  // static shared variables take the rest
 
 // Shared-memory layout for a launch with per-pipeline lists of kcap entries.
 void layout_smem(const Params& P, TcArgs& T, int kcap) {
@@ -853,14 +866,18 @@ void layout_smem(const Params& P, TcArgs& T, int kcap) {
   T.sm_xw = o; o += round_up(sumK * T.kw * 4, 16);
   T.sm_dem = o; o += sumK * 16;
   T.sm_rows = o; o += T.pipes * 2 * MF_MAX_MODELS * 128;  // byte digits of two tiles per pipeline
-  T.sm_topk = o; o += kcap > 0 ? (uint32_t)(T.pipes * topk_bytes_pipe(kcap)) : 0u;
+  // the candidate queue: 512 entries (a merge every few tiles) where shared memory allows,
+  // else one tile's 128 (a merge after every tile that queued a candidate)
+  const uint32_t rest = o + 16 + 8 * (3 + 2 * kTcMaxPipes);
+  T.qcap = 128;
+  if (kcap > 0 && rest + T.pipes * topk_bytes_pipe(kcap, 512) <= kSmemLimit) T.qcap = 512;
+  T.sm_topk = o; o += kcap > 0 ? (uint32_t)(T.pipes * topk_bytes_pipe(kcap, T.qcap)) : 0u;
   o = round_up((int)o, 16);
   T.sm_bar = o; o += 8 * (3 + 2 * kTcMaxPipes);
   T.sm_total = o;
   T.kcap = kcap;
 }
 
-constexpr uint32_t kSmemLimit = 227 * 1024 - 1024;  // static shared variables take the rest
 constexpr size_t kPassImageBudget = 160 * 1024;      // bf16 weights staged per pass
 
 using TcFn = void (*)(const Params, const TcArgs, const RangeArgs, const TcList);

@@ -55,6 +55,7 @@ struct TcArgs {
   uint32_t sm_xw, sm_dem, sm_rows, sm_topk, sm_bar, sm_total;  // shared-memory byte offsets
   uint32_t img_model;                 // bytes of one model's B1 + B2 + B3 images
   int32_t kcap;                       // per-pipeline list length the layout was sized for
+  int32_t qcap;                       // per-pipeline candidate queue (128 or 512, a power of two)
   uint32_t step[MF_MAX_MODELS];       // mixed-radix digits of the per-tile index stride (range mode)
   // models whose weights do not fit shared memory together run in passes of consecutive
   // models [pass_m[p], pass_m[p + 1]); each pass's image is staged on its own
