@@ -141,6 +141,12 @@ __device__ __forceinline__ uint32_t bf16_bits(float v) {
   return (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v));
 }
 
+__device__ __forceinline__ uint32_t tmem_ld_x1(uint32_t taddr) {
+  uint32_t r;
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];" : "=r"(r) : "r"(taddr));
+  return r;
+}
+
 __device__ __forceinline__ void tmem_ld_x16(uint32_t taddr, uint32_t (&r)[16]) {
   asm volatile("tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
                : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
@@ -547,8 +553,8 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     else tmem_st_x16(tA + lane_off, v);
   };
   // Digits of tile `tile` into buffer dg (range mode: `from`, the previous tile's digits,
-  // stepped by the tile stride) and its first A1 row (model m0) with the aggregate words.
-  auto load_tile = [&](uint64_t tile, uint8_t* dg, const uint8_t* from) {
+  // stepped by the tile stride).
+  auto tile_digits = [&](uint64_t tile, uint8_t* dg, const uint8_t* from) {
     const uint64_t t = tile * 128 + row;
     if (MODE == kTcRange) {
       if (from == nullptr) {
@@ -573,7 +579,9 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
       }
       for (int i = 0; i < N; ++i) dg[i * 128 + row] = (uint8_t)digit_of(P, idx, i);
     }
-    // aggregate state (fp32, model order) and its bf16 hi/lo words
+  };
+  // The aggregate state of a tile (fp32, model order) as the A1 words: bf16 hi/lo pairs.
+  auto tile_agg = [&](const uint8_t* dg) -> uint4 {
     float A0 = 0.f, A1 = 0.f, A2 = 0.f;
 #pragma unroll (NM > 0 ? NM : 1)
     for (int i = 0; i < N; ++i) {
@@ -585,7 +593,12 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     const uint32_t l0 = bf16_bits(v0 - __uint_as_float(h0 << 16));
     const uint32_t l1 = bf16_bits(v1 - __uint_as_float(h1 << 16));
     const uint32_t l2 = bf16_bits(v2 - __uint_as_float(h2 << 16));
-    write_a1(m0, dg, true, make_uint4(h0 | (h1 << 16), h2 | (0x3F80u << 16) /* bf16 1.0 */, l0 | (l1 << 16), l2));
+    return make_uint4(h0 | (h1 << 16), h2 | (0x3F80u << 16) /* bf16 1.0 */, l0 | (l1 << 16), l2);
+  };
+  // Digits of tile `tile` and its first A1 row (model m0) with the aggregate words.
+  auto load_tile = [&](uint64_t tile, uint8_t* dg, const uint8_t* from) {
+    tile_digits(tile, dg, from);
+    write_a1(m0, dg, true, tile_agg(dg));
   };
   // the model-i A1 row of the current tile (aggregate words already in place when AWO >= 0)
   auto next_a1 = [&](int i, const uint8_t* dg) {
@@ -606,9 +619,45 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     }
   };
 
-  // ---- objective, constraints and top-k of a finished tile from its layer-3 outputs ----
-  constexpr int D3W = N3 == 16 ? 16 : 32;
-  auto finish_tile = [&](const uint32_t (&d3)[D3W], uint64_t tile_f, const uint8_t* dg) {
+  // ---- objective and constraints, model by model, from the layer-3 outputs ----
+  // Model j's two outputs (columns j and n3/2 + j of D3) are read once its layer 3 has
+  // landed, and its terms join this thread's running objective for the tile; later
+  // models' layer-3 MMAs add zero to those columns.
+  const int half3 = N3 == 16 ? 8 : (T.n3 >> 1);
+  float acc_J = 0.f, acc_pen = 0.f;
+  bool acc_ok = true, acc_near = true;
+  auto add_model = [&](int j, const uint8_t* dg, uint64_t tile_f) {
+    const uint32_t a = tmem_ld_x1(tD3 + lane_off + (uint32_t)j);
+    const uint32_t b = tmem_ld_x1(tD3 + lane_off + (uint32_t)(half3 + j));
+    tmem_wait_ld();
+    const float thr = tc_out(P, __uint_as_float(a) + s_b3[j][0]);
+    const float lat = tc_out(P, __uint_as_float(b) + s_b3[j][1]);
+    if (MODE == kTcList && L.pred) {
+      const uint64_t t = tile_f * 128 + row;
+      if (t < n && L.idx[t] < P.total) {
+        L.pred[(t * N + j) * 2 + 0] = thr;
+        L.pred[(t * N + j) * 2 + 1] = lat;
+      }
+    }
+    if (UT) {  // Eq. 3 utility, floors f >= tau
+      float f;
+      acc_J += util_term(P, j, P.off[j] + dg[j * 128 + row], thr, &f);
+      const float tau = P.u_tau[j];
+      acc_ok = acc_ok && (f >= tau);
+      acc_near = acc_near && (f >= tau - 2e-2f * fmaxf(fabsf(tau), fabsf(f)));
+      return;
+    }
+    acc_J = fmaf(P.w[j], thr, acc_J);
+    const float sla = P.sla[j];
+    acc_ok = acc_ok && (lat <= sla);
+    // shortlist test: within the bf16 error band of the ceiling
+    acc_near = acc_near && (lat <= sla + 2e-2f * fmaxf(fabsf(sla), fabsf(lat)));
+    const float over = lat - sla;
+    acc_pen += over > 0.f ? over : 0.f;
+  };
+  // The end of a tile whose every model has been added: the VRAM bound, the earlier
+  // passes' record, feasibility, the count and the top-k queue; then a fresh objective.
+  auto finish_tile = [&](uint64_t tile_f, const uint8_t* dg) {
     const uint64_t t = tile_f * 128 + row;
     bool valid = t < n;
     uint64_t idx;
@@ -621,38 +670,12 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     float vram = 0.f;  // the candidate's summed VRAM demand (model order, as the aggregate)
 #pragma unroll (NM > 0 ? NM : 1)
     for (int i = 0; i < N; ++i) vram += dem_s[P.off[i] + dg[i * 128 + row]].y;
-    float J = 0.f, pen = 0.f;
-    bool sla_ok = true, sla_near = true;
-    const int half3 = T.n3 >> 1;  // thr of model i in column i, lat in column half3 + i
-    constexpr int MU = N3 == 16 ? 8 : 16;  // a 16-column layer-3 tile holds at most 8 models
-#pragma unroll
-    for (int i = 0; i < MU; ++i) {
-      if (i >= m1) break;
-      if (i < m0) continue;
-      const float thr = tc_out(P, __uint_as_float(d3[i]) + s_b3[i][0]);
-      const float lat = tc_out(P, __uint_as_float(N3 == 16 ? d3[(8 + i) & 15]
-                                                : half3 == 8 ? d3[(8 + i) & (D3W - 1)] : d3[(16 + i) & (D3W - 1)]) +
-                                  s_b3[i][1]);
-      if (MODE == kTcList && valid && L.pred) {
-        L.pred[(t * N + i) * 2 + 0] = thr;
-        L.pred[(t * N + i) * 2 + 1] = lat;
-      }
-      if (UT) {  // Eq. 3 utility, floors f >= tau
-        float f;
-        J += util_term(P, i, P.off[i] + dg[i * 128 + row], thr, &f);
-        const float tau = P.u_tau[i];
-        sla_ok = sla_ok && (f >= tau);
-        sla_near = sla_near && (f >= tau - 2e-2f * fmaxf(fabsf(tau), fabsf(f)));
-        continue;
-      }
-      J = fmaf(P.w[i], thr, J);
-      const float sla = P.sla[i];
-      sla_ok = sla_ok && (lat <= sla);
-      // shortlist test: within the bf16 error band of the ceiling
-      sla_near = sla_near && (lat <= sla + 2e-2f * fmaxf(fabsf(sla), fabsf(lat)));
-      const float over = lat - sla;
-      pen += over > 0.f ? over : 0.f;
-    }
+    float J = acc_J, pen = acc_pen;
+    bool sla_ok = acc_ok, sla_near = acc_near;
+    acc_J = 0.f;
+    acc_pen = 0.f;
+    acc_ok = true;
+    acc_near = true;
     if (MP && !T.pass_first && t < n) {  // the earlier passes' models
       const float4 pr = T.partial[t];
       J += pr.x;
@@ -694,21 +717,6 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
       if (*(volatile int*)tk.qn > T.qcap - 128) tc_topk_merge(tk, row, barid);
     }
   };
-  auto load_d3 = [&](uint32_t (&d3)[D3W]) {
-    if constexpr (N3 == 16) {
-      tmem_ld_x16(tD3 + lane_off, d3);
-    } else if (T.n3 == 16) {
-      uint32_t r16[16];
-      tmem_ld_x16(tD3 + lane_off, r16);
-      tmem_wait_ld();
-#pragma unroll
-      for (int j = 0; j < 16; ++j) d3[j] = r16[j];
-    } else {
-      tmem_ld_x32(tD3 + lane_off, d3);
-    }
-    tmem_wait_ld();
-  };
-
   uint64_t tile = gpipe;
   int buf = 0;
   if (tile * 128 < n) load_tile(tile, digits, nullptr);
@@ -722,12 +730,32 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   // the previous tile is finished once its last layer 3 (issued in this tile's first
   // round A) has landed
   bool pending = false;
-  uint32_t d3[D3W];
+  // the next tile's digits, aggregate and first A1 row are prepared in stages, each
+  // while one model's layer 2 runs
+  const int st_dig = m0 + 1 < m1 ? m0 + 1 : m1 - 1;
+  const int st_agg = m0 + 2 < m1 ? m0 + 2 : m1 - 1;
+  uint4 aw_nx = make_uint4(0u, 0u, 0u, 0u);
 
   for (; tile * 128 < n; tile += gstride) {
     uint8_t* dg = digits + buf * (MF_MAX_MODELS * 128);
     uint8_t* dg_p = digits + (buf ^ 1) * (MF_MAX_MODELS * 128);
     const bool has_next = (tile + gstride) * 128 < n;
+    // Work off the critical path, while layer 2 of model i runs (or, with one hidden
+    // layer, after its layer-1 epilogue): the objective terms of the model whose layer 3
+    // has landed (at the first model: the previous tile's last, and that tile's end),
+    // a stage of the next tile, the next A1 row.
+    auto side_work = [&](int i) {
+      if (i > m0) {
+        add_model(i - 1, dg, tile);
+      } else if (pending) {
+        add_model(m1 - 1, dg_p, tile - gstride);
+        finish_tile(tile - gstride, dg_p);
+      }
+      if (has_next && i == st_dig) tile_digits(tile + gstride, dg_p, dg);
+      if (has_next && i == st_agg) aw_nx = tile_agg(dg_p);
+      if (i + 1 < m1) next_a1(i + 1, dg);
+      else if (has_next) write_a1(m0, dg_p, true, aw_nx);
+    };
 #pragma unroll (NM > 0 ? NM : 1)
     for (int i = m0; i < m1; ++i) {
       const bool l3 = i > m0 || pending;
@@ -741,15 +769,10 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
       }
       await_a();
       hidden_epilogue<(S2 > 0 ? (S2 - 1) * 16 : 0)>(T.h1, tD + lane_off, tH1 + lane_off, []() {}, [&]() {
-        if (l3) {
-          await_b();
-          if (i == m0) load_d3(d3);  // the previous tile's outputs, before layer 3 restarts
-        }
+        if (l3) await_b();  // the previous model's layer 3 has read H
       });
       if (T.h2 == 0) {  // one hidden layer: no round B
-        if (i == m0 && pending) finish_tile(d3, tile - gstride, dg_p);
-        if (i + 1 < m1) next_a1(i + 1, dg);
-        else if (has_next) load_tile(tile + gstride, dg_p, dg);
+        side_work(i);
         if (next_l1) issue_next_l1(inext);
         publish();
         continue;
@@ -761,9 +784,7 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
         issue_mma2(i);
         mma_commit_warp(barA);
       }
-      if (i == m0 && pending) finish_tile(d3, tile - gstride, dg_p);
-      if (i + 1 < m1) next_a1(i + 1, dg);
-      else if (has_next) load_tile(tile + gstride, dg_p, dg);  // next tile: digits, aggregate, A1
+      side_work(i);
       await_a();
       hidden_epilogue<(S3 > 0 ? S3 * 16 : 0)>(
           T.h2, tD + lane_off, tH2 + lane_off,
@@ -783,8 +804,9 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
       mma_commit_warp(barB);
     }
     await_b();
-    load_d3(d3);
-    finish_tile(d3, tile - gstride, digits + (buf ^ 1) * (MF_MAX_MODELS * 128));
+    uint8_t* dg_last = digits + (buf ^ 1) * (MF_MAX_MODELS * 128);
+    add_model(m1 - 1, dg_last, tile - gstride);
+    finish_tile(tile - gstride, dg_last);
   }
   if (MODE == kTcRange && (!MP || T.pass_last)) {  // what is still queued joins the list
     const CtaTopK tk = topk();
