@@ -183,6 +183,11 @@ __device__ __forceinline__ void tmem_st_x16(uint32_t taddr, const uint32_t (&v)[
 // ---------------------------------------------------------------------------
 enum { kTcRange = 0, kTcList = 1 };
 constexpr int kTcMaxPipes = 4;
+// Each 128-row pipeline has four epilogue warps (warp w reaches tensor-memory lanes
+// 32 (w % 4) ..) and one warp that issues its MMAs: warps [0, 4 pipes) are the epilogue
+// warps (pipeline w / 4), warps [4 pipes, 5 pipes) the issuing warps (pipeline w - 4 pipes,
+// so the issuers sit on different schedulers).
+constexpr int kTcPipeThreads = 160;
 constexpr uint32_t kWaitLimit = 4096;  // suspended retries (~1 ms each at most)
 
 struct TcList {
@@ -286,7 +291,7 @@ __device__ __forceinline__ void mma_steps(int steps, uint32_t d_tmem, uint32_t a
 // Hidden epilogue: fp32 accumulators [0, width) at `src` -> ReLU -> bf16 pairs at `dst`.
 // 64 columns are loaded before one wait.  `after_load` runs once the last accumulator
 // column is in registers (the accumulator columns are then free for the next layer);
-// `before_store` runs once, before the first stores (round A waits there for the
+// `before_store` runs once, before the first stores (the layer-1 epilogue waits there for the
 // previous model's layer 3, which reads the same tensor-memory columns).
 template <int W, class FL, class FS>
 __device__ __forceinline__ void hidden_epilogue(int width, uint32_t src, uint32_t dst, FL after_load,
@@ -331,16 +336,19 @@ __device__ __forceinline__ void hidden_epilogue(int width, uint32_t src, uint32_
 // compile time (0: run time); the per-model loop is then unrolled, so every per-model
 // offset, descriptor and branch is a constant.
 //
-// Per 128-row pipeline and model i the work is two rounds of MMAs:
-//   round A: layer 1 of model i (commit A) and layer 3 of model i - 1 (commit B; the
-//            last model's layer 3 of a tile rides in the next tile's first round A);
-//            epilogue: D1 -> H1, stored once layer 3 has finished reading H
-//   round B: layer 2 of model i (commit A); while it runs the next model's A1 is
-//            written (at the last model: the next tile's digits, aggregate and A1), and
-//            at the first model the previous tile's objective, constraints and top-k
-//            are finished from its layer-3 outputs; epilogue: D2 -> H2.
+// Per 128-row pipeline and model i, the issuing warp runs three MMA groups, each on a
+// hand-off (named barrier) from the pipeline's four epilogue warps:
+//   H1 stored     -> layer 2 of model i (commit A)
+//   D2 read, the next A1 row written -> layer 1 of model i + 1, or of the next tile's
+//                    first model (commit A)
+//   H2 stored     -> layer 3 of model i (commit B)
+// and the epilogue warps, per model: D1 -> H1 (stored once the previous layer 3 has read
+// H); while layer 2 runs, the objective terms of the previous model (at the first model:
+// the previous tile's last, and that tile's constraints and top-k), a stage of the next
+// tile's digits and aggregate, and the next A1 row; then D2 -> H2.  The issuing warp does
+// nothing else, so an MMA group starts as soon as its operands are stored.
 template <int MODE, int KW, int AWO, int S1, int S2, int S3, int N3, bool MP, bool UT, int NM>
-__global__ void __launch_bounds__(kTcMaxPipes * 128, 1)
+__global__ void __launch_bounds__(kTcMaxPipes * kTcPipeThreads, 1)
 k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   static_assert(AWO < 0 || AWO == 4 || AWO == 8, "partial A1 rows are written for these layouts only");
   extern __shared__ __align__(1024) unsigned char smem[];
@@ -358,10 +366,11 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   // and keeps everything derived from it (pipeline, tensor-memory addresses, issuer roles)
   // in uniform registers with uniform branches
   const int warp = __shfl_sync(0xffffffffu, tid >> 5, 0), lane = tid & 31;
-  const int pipe = warp >> 2, wq = warp & 3;
-  const int row = wq * 32 + lane;
   const int N = NM > 0 ? NM : P.n_models;
   const int npipes = T.pipes;
+  const bool issuer = warp >= 4 * npipes;  // the pipeline's MMA-issuing warp
+  const int pipe = issuer ? warp - 4 * npipes : warp >> 2, wq = warp & 3;
+  const int row = wq * 32 + lane;
 
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + T.sm_bar);
   const uint4* xw_s = reinterpret_cast<const uint4*>(smem + T.sm_xw);
@@ -374,7 +383,7 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     s_abort = 0;
     for (int j = 0; j < 1 + 2 * npipes; ++j) mbar_init(&bars[j], 1);
     mbar_init(&bars[1 + 2 * npipes], 1);           // the timeout test's barrier: nothing arrives
-    mbar_init(&bars[2 + 2 * npipes], 2 * npipes);  // drain: one commit per issuing warp
+    mbar_init(&bars[2 + 2 * npipes], npipes);  // drain: one commit per issuing warp
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 0) {
@@ -423,7 +432,7 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     tk.k = kcap;
     return tk;
   };
-  if (MODE == kTcRange) {
+  if (MODE == kTcRange && !issuer) {
     const CtaTopK tk = topk();
     const size_t gl = ((size_t)blockIdx.x * npipes + pipe) * kcap;
     for (int e = row; e < kcap; e += 128) {
@@ -443,26 +452,22 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   const uint32_t tD = tp + T.col_d, tA = tp + T.col_a, tD3 = tp + T.col_d3, tOnes = tp + T.col_ones;
   const uint32_t tH1 = tOnes - (uint32_t)(T.h1 / 2);                        // layer-2 A operand
   const uint32_t tH2 = T.h2 > 0 ? tOnes - (uint32_t)(T.h2 / 2) : tH1;       // layer-3 A operand
-  // Layers 1 and 2 of pipeline p are issued by its warp p (warp 4p + p of the CTA), layer 3
-  // by its warp p + 1: each scheduler's MMA queue serves one pipeline's layers 1-2 and
-  // another's layer 3, and a pipeline's layer 3 does not queue behind its layer 1.
-  const bool issuer = (wq == (pipe & 3));
-  const bool issuer3 = (wq == ((pipe + 1) & 3));
-  uint64_t* barA = &bars[1 + 2 * pipe];
-  uint64_t* barB = &bars[2 + 2 * pipe];
+  uint64_t* barA = &bars[1 + 2 * pipe];  // layers 1 and 2 completed (alternating)
+  uint64_t* barB = &bars[2 + 2 * pipe];  // layer 3 completed
   uint32_t phA = 0, phB = 0;
-  const int barid = 1 + pipe;
-  const int barid_d = 1 + npipes + pipe;  // "accumulators read": the issuing warp syncs, the rest arrive
+  // epilogue -> issuer hand-offs alternate between two named barriers per pipeline (the
+  // epilogue warps arrive, the issuing warp syncs; the epilogue warps never run two
+  // hand-offs ahead); the pipeline's top-k uses a third among its epilogue warps
+  const int sig0 = 1 + 2 * pipe, barid = 1 + 2 * npipes + pipe;
   const uint32_t id1 = idesc_bf16(T.h1), id2 = idesc_bf16(T.h2), id3 = idesc_bf16(T.n3);
   const int s1 = T.k1 / 16, s2 = T.h1 / 16 + 1, s3 = T.hl / 16;
   const int m0 = MP ? T.m0 : 0, m1 = MP ? T.m1 : N;  // this pass's models
   const float vcap = P.vram_cap;
-  {  // constant ones block: word 0 = (1, 1) feeds the bias hi/lo rows of B2
+  if (!issuer) {  // constant ones block: word 0 = (1, 1) feeds the bias hi/lo rows of B2
     uint32_t v[8] = {0x3F803F80u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
     tmem_st_x8(tOnes + lane_off, v);
   }
   if (P.wait_test) mbar_wait_test(&bars[1 + 2 * npipes], P.wait_test, &s_abort, P.status);
-  wait_bar(&bars[0], 0);  // weights landed
 
   unsigned int my_count = 0;
 
@@ -487,11 +492,10 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     mma_steps<S3>(s3, tD3, tH2, smem_desc(sb3 + (uint32_t)(i - m0) * T.img_model, 128u, (uint32_t)(T.hl / 8) * 128u),
                   id3, i > m0 ? 1u : 0u);
   };
-  // Every warp waits on the commit's mbarrier itself (suspended until the phase completes).
+  // The epilogue warps wait on the commits' mbarriers (suspended until the phase completes).
   auto await_a = [&]() {
-    if (issuer) wait_bar(barA, phA);
+    wait_bar(barA, phA);
     phA ^= 1u;
-    named_bar(barid, 128);
     tc_fence_after();
   };
   auto await_b = [&]() {
@@ -499,24 +503,20 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     phB ^= 1u;
     tc_fence_after();
   };
-  auto publish = [&]() {  // make this thread's tensor-memory stores visible to the issuer
+  uint32_t ksig = 0;
+  // epilogue warps: this thread's tensor-memory loads and stores so far are complete and
+  // ordered before the issuing warp's next MMAs
+  auto signal = [&]() {
     tmem_wait_st();
     tc_fence_before();
-    named_bar(barid, 128);
+    named_arrive(sig0 + (int)(ksig & 1u), 160);
+    ++ksig;
   };
-  // The accumulators have been read and the next A1 row written: the issuing warp starts
-  // the next layer 1 while the others go on converting.
-  auto issue_next_l1 = [&](int inext) {
-    tmem_wait_st();
-    tc_fence_before();
-    if (issuer) {
-      named_bar(barid_d, 128);
-      tc_fence_after();
-      issue_mma1(inext);
-      mma_commit_warp(barA);
-    } else {
-      named_arrive(barid_d, 128);
-    }
+  // issuing warp: the epilogue warps' next hand-off
+  auto take = [&]() {
+    named_bar(sig0 + (int)(ksig & 1u), 160);
+    ++ksig;
+    tc_fence_after();
   };
 
   // ---- A1 rows: [local features | aggregate hi | 1 | aggregate lo] ----
@@ -717,104 +717,115 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
       if (*(volatile int*)tk.qn > T.qcap - 128) tc_topk_merge(tk, row, barid);
     }
   };
-  uint64_t tile = gpipe;
-  int buf = 0;
-  if (tile * 128 < n) load_tile(tile, digits, nullptr);
-  publish();  // ones block and the first A1
-  if (tile * 128 < n && issuer) {  // the first layer 1; every later one starts in the round before
-    tc_fence_after();
-    issue_mma1(m0);
-    mma_commit_warp(barA);
-  }
-
-  // the previous tile is finished once its last layer 3 (issued in this tile's first
-  // round A) has landed
-  bool pending = false;
-  // the next tile's digits, aggregate and first A1 row are prepared in stages, each
-  // while one model's layer 2 runs
-  const int st_dig = m0 + 1 < m1 ? m0 + 1 : m1 - 1;
-  const int st_agg = m0 + 2 < m1 ? m0 + 2 : m1 - 1;
-  uint4 aw_nx = make_uint4(0u, 0u, 0u, 0u);
-
-  for (; tile * 128 < n; tile += gstride) {
-    uint8_t* dg = digits + buf * (MF_MAX_MODELS * 128);
-    uint8_t* dg_p = digits + (buf ^ 1) * (MF_MAX_MODELS * 128);
-    const bool has_next = (tile + gstride) * 128 < n;
-    // Work off the critical path, while layer 2 of model i runs (or, with one hidden
-    // layer, after its layer-1 epilogue): the objective terms of the model whose layer 3
-    // has landed (at the first model: the previous tile's last, and that tile's end),
-    // a stage of the next tile, the next A1 row.
-    auto side_work = [&](int i) {
-      if (i > m0) {
-        add_model(i - 1, dg, tile);
-      } else if (pending) {
-        add_model(m1 - 1, dg_p, tile - gstride);
-        finish_tile(tile - gstride, dg_p);
-      }
-      if (has_next && i == st_dig) tile_digits(tile + gstride, dg_p, dg);
-      if (has_next && i == st_agg) aw_nx = tile_agg(dg_p);
-      if (i + 1 < m1) next_a1(i + 1, dg);
-      else if (has_next) write_a1(m0, dg_p, true, aw_nx);
-    };
+  if (issuer) {
+    // ---- the issuing warp: one MMA group per hand-off of the epilogue warps ----
+    wait_bar(&bars[0], 0);  // weights landed
+    uint64_t tile = gpipe;
+    if (tile * 128 < n) {
+      take();  // the first A1 row
+      issue_mma1(m0);
+      mma_commit_warp(barA);
+    }
+    for (; tile * 128 < n; tile += gstride) {
+      const bool has_next = (tile + gstride) * 128 < n;
 #pragma unroll (NM > 0 ? NM : 1)
-    for (int i = m0; i < m1; ++i) {
-      const bool l3 = i > m0 || pending;
-      const bool next_l1 = i + 1 < m1 || has_next;
-      const int inext = i + 1 < m1 ? i + 1 : m0;
-      // ---- round A: layer 1 of model i (already issued), layer 3 of the model before ----
-      if (issuer3 && l3) {
-        tc_fence_after();
-        issue_mma3(i > m0 ? i - 1 : m1 - 1);
+      for (int i = m0; i < m1; ++i) {
+        const bool next_l1 = i + 1 < m1 || has_next;
+        if (T.h2 > 0) {
+          take();  // H1 of model i stored
+          issue_mma2(i);
+          mma_commit_warp(barA);
+        }
+        if (next_l1) {
+          take();  // accumulators read, the next A1 row written
+          issue_mma1(i + 1 < m1 ? i + 1 : m0);
+          mma_commit_warp(barA);
+        }
+        take();  // the last hidden layer of model i stored
+        issue_mma3(i);
         mma_commit_warp(barB);
       }
-      await_a();
-      hidden_epilogue<(S2 > 0 ? (S2 - 1) * 16 : 0)>(T.h1, tD + lane_off, tH1 + lane_off, []() {}, [&]() {
-        if (l3) await_b();  // the previous model's layer 3 has read H
-      });
-      if (T.h2 == 0) {  // one hidden layer: no round B
+    }
+  } else {
+    // ---- the epilogue warps ----
+    uint64_t tile = gpipe;
+    int buf = 0;
+    if (tile * 128 < n) {
+      load_tile(tile, digits, nullptr);
+      signal();  // ones block and the first A1 row
+    }
+    // the previous tile is finished once its last layer 3 (issued at the end of that
+    // tile) has landed, during this tile's first model
+    bool pending = false;
+    // the next tile's digits, aggregate and first A1 row are prepared in stages, each
+    // while one model's layer 2 runs
+    const int st_dig = m0 + 1 < m1 ? m0 + 1 : m1 - 1;
+    const int st_agg = m0 + 2 < m1 ? m0 + 2 : m1 - 1;
+    uint4 aw_nx = make_uint4(0u, 0u, 0u, 0u);
+    for (; tile * 128 < n; tile += gstride) {
+      uint8_t* dg = digits + buf * (MF_MAX_MODELS * 128);
+      uint8_t* dg_p = digits + (buf ^ 1) * (MF_MAX_MODELS * 128);
+      const bool has_next = (tile + gstride) * 128 < n;
+      // Work off the critical path, while layer 2 of model i runs (or, with one hidden
+      // layer, after its layer-1 epilogue): the objective terms of the model whose layer
+      // 3 has landed (at the first model: the previous tile's last, and that tile's end),
+      // a stage of the next tile, the next A1 row.
+      auto side_work = [&](int i) {
+        if (i > m0) {
+          add_model(i - 1, dg, tile);
+        } else if (pending) {
+          add_model(m1 - 1, dg_p, tile - gstride);
+          finish_tile(tile - gstride, dg_p);
+        }
+        if (has_next && i == st_dig) tile_digits(tile + gstride, dg_p, dg);
+        if (has_next && i == st_agg) aw_nx = tile_agg(dg_p);
+        if (i + 1 < m1) next_a1(i + 1, dg);
+        else if (has_next) write_a1(m0, dg_p, true, aw_nx);
+      };
+#pragma unroll (NM > 0 ? NM : 1)
+      for (int i = m0; i < m1; ++i) {
+        const bool l3 = i > m0 || pending;
+        const bool next_l1 = i + 1 < m1 || has_next;
+        // ---- layer 1 of model i landed: D1 -> H1 ----
+        await_a();
+        hidden_epilogue<(S2 > 0 ? (S2 - 1) * 16 : 0)>(T.h1, tD + lane_off, tH1 + lane_off, []() {}, [&]() {
+          if (l3) await_b();  // the previous model's layer 3 has read H
+        });
+        if (T.h2 == 0) {  // one hidden layer: the next layer 1, then layer 3 of model i
+          side_work(i);
+          if (next_l1) signal();
+          signal();
+          continue;
+        }
+        signal();  // H1 stored: layer 2 of model i
         side_work(i);
-        if (next_l1) issue_next_l1(inext);
-        publish();
-        continue;
+        // ---- layer 2 of model i landed: D2 -> H2 ----
+        await_a();
+        hidden_epilogue<(S3 > 0 ? S3 * 16 : 0)>(
+            T.h2, tD + lane_off, tH2 + lane_off,
+            [&]() {
+              if (next_l1) signal();  // accumulators read, next A1 written: the next layer 1
+            },
+            []() {});
+        signal();  // H2 stored: layer 3 of model i
       }
-      publish();
-      // ---- round B: layer 2 of model i ----
-      if (issuer) {
-        tc_fence_after();
-        issue_mma2(i);
-        mma_commit_warp(barA);
-      }
-      side_work(i);
-      await_a();
-      hidden_epilogue<(S3 > 0 ? S3 * 16 : 0)>(
-          T.h2, tD + lane_off, tH2 + lane_off,
-          [&]() {
-            if (next_l1) issue_next_l1(inext);
-          },
-          []() {});
-      publish();
+      pending = true;
+      buf ^= 1;
     }
-    pending = true;
-    buf ^= 1;
-  }
-  if (pending) {  // the last tile's last layer 3
-    if (issuer3) {
-      tc_fence_after();
-      issue_mma3(m1 - 1);
-      mma_commit_warp(barB);
+    if (pending) {  // the last tile's last layer 3
+      await_b();
+      uint8_t* dg_last = digits + (buf ^ 1) * (MF_MAX_MODELS * 128);
+      add_model(m1 - 1, dg_last, tile - gstride);
+      finish_tile(tile - gstride, dg_last);
     }
-    await_b();
-    uint8_t* dg_last = digits + (buf ^ 1) * (MF_MAX_MODELS * 128);
-    add_model(m1 - 1, dg_last, tile - gstride);
-    finish_tile(tile - gstride, dg_last);
   }
-  if (MODE == kTcRange && (!MP || T.pass_last)) {  // what is still queued joins the list
+  if (MODE == kTcRange && (!MP || T.pass_last) && !issuer) {  // what is still queued joins the list
     const CtaTopK tk = topk();
     named_bar(barid, 128);
     if (*(volatile int*)tk.qn > 0) tc_topk_merge(tk, row, barid);
   }
 
-  if (MODE == kTcRange && (!MP || T.pass_last)) {
+  if (MODE == kTcRange && (!MP || T.pass_last) && !issuer) {
     const CtaTopK tk = topk();
     const size_t gl = ((size_t)blockIdx.x * npipes + pipe) * kcap;
     for (int e = row; e < kcap; e += 128) {
@@ -829,7 +840,7 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   // Nothing of this CTA may still run when its tensor memory is freed: each issuing warp
   // commits its MMAs to the drain barrier, and everyone waits for them and for the weight
   // copy (after a wait that gave up, these are the only waits still made).
-  if (issuer || issuer3) mma_commit_warp(&bars[2 + 2 * npipes]);
+  if (issuer) mma_commit_warp(&bars[2 + 2 * npipes]);
   mbar_wait_drain(&bars[2 + 2 * npipes], 0, P.status);
   mbar_wait_drain(&bars[0], 0, P.status);
   tc_fence_before();
@@ -1145,7 +1156,7 @@ mf_status tc_search_chunk(mf_ctx* c, const RangeArgs& a, cudaStream_t s, int* nl
     r.first = a.first && b == 0;
     for (int p = 0; p < T.npasses; ++p) {
       set_pass(T, p, partial);
-      tc_kernel(kTcRange, T, c->P.objective == MF_OBJ_UTILITY, c->P.n_models)<<<c->num_sms, T.pipes * 128, smem, s>>>(c->P, T, r, L);
+      tc_kernel(kTcRange, T, c->P.objective == MF_OBJ_UTILITY, c->P.n_models)<<<c->num_sms, T.pipes * kTcPipeThreads, smem, s>>>(c->P, T, r, L);
       MF_CUDA(cudaGetLastError());
       ++launches;
     }
@@ -1175,7 +1186,7 @@ mf_status tc_score_list(mf_ctx* c, const uint64_t* idx, uint64_t n, float* score
     TcList L{idx + b, m, score + b, feas ? feas + b : nullptr, pred ? pred + b * N * 2 : nullptr};
     for (int p = 0; p < T.npasses; ++p) {
       set_pass(T, p, partial);
-      tc_kernel(kTcList, T, c->P.objective == MF_OBJ_UTILITY, c->P.n_models)<<<(unsigned)grid, T.pipes * 128, smem, s>>>(c->P, T, R, L);
+      tc_kernel(kTcList, T, c->P.objective == MF_OBJ_UTILITY, c->P.n_models)<<<(unsigned)grid, T.pipes * kTcPipeThreads, smem, s>>>(c->P, T, R, L);
       MF_CUDA(cudaGetLastError());
     }
   }
