@@ -35,6 +35,7 @@
 #include <cuda_bf16.h>
 
 #include <cstring>
+#include <type_traits>
 #include <vector>
 
 #include "mf_internal.cuh"
@@ -81,6 +82,11 @@ __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence:
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 __device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+// wait for this thread's tensor-memory loads; the two registers loaded last are tied to
+// the wait, so no use of them is scheduled before it
+__device__ __forceinline__ void tmem_wait_ld_2(uint32_t& a, uint32_t& b) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" : "+r"(a), "+r"(b)::"memory");
+}
 
 __device__ __forceinline__ void named_bar(int id, int nthreads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
@@ -351,6 +357,12 @@ template <int MODE, int KW, int AWO, int S1, int S2, int S3, int N3, bool MP, bo
 __global__ void __launch_bounds__(kTcMaxPipes * kTcPipeThreads, 1)
 k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   static_assert(AWO < 0 || AWO == 4 || AWO == 8, "partial A1 rows are written for these layouts only");
+  static_assert(NM <= 7, "packed digits hold at most seven models");
+  // With the model count fixed at compile time (range mode), a tile's digits live in
+  // registers, packed one per byte (model N - 1 in the lowest byte); otherwise in shared
+  // memory, one byte per model and row, two tiles.
+  constexpr bool RD = NM > 0 && MODE == kTcRange;
+  using DS = typename std::conditional<RD, uint64_t, uint8_t*>::type;
   extern __shared__ __align__(1024) unsigned char smem[];
   __shared__ uint32_t s_tmem;
   __shared__ int s_abort;
@@ -524,8 +536,13 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   // tile's first A1 row, and the later models rewrite only the local-feature words (when
   // the aggregate's position is a compile-time constant).
   const int awo = AWO >= 0 ? AWO : (T.dle >> 1);
-  auto write_a1 = [&](int i, const uint8_t* dg, bool with_agg, uint4 aw4) {
-    const uint4* src = xw_s + (size_t)(P.off[i] + dg[i * 128 + row]) * (KW >> 2);
+  // digit of model i in a digit set
+  auto dig = [&](DS ds, int i) -> uint32_t {
+    if constexpr (RD) return (uint32_t)(ds >> (8 * (NM - 1 - i))) & 0xFFu;
+    else return ds[i * 128 + row];
+  };
+  auto write_a1 = [&](int i, DS dg, bool with_agg, uint4 aw4) {
+    const uint4* src = xw_s + (size_t)(P.off[i] + dig(dg, i)) * (KW >> 2);
     if (AWO >= 0 && !with_agg) {
       uint32_t v[AWO > 0 ? AWO : 1];
 #pragma unroll
@@ -552,15 +569,31 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     if constexpr (KW == 8) tmem_st_x8(tA + lane_off, v);
     else tmem_st_x16(tA + lane_off, v);
   };
-  // Digits of tile `tile` into buffer dg (range mode: `from`, the previous tile's digits,
-  // stepped by the tile stride).
-  auto tile_digits = [&](uint64_t tile, uint8_t* dg, const uint8_t* from) {
+  // Digits of tile `tile` (in shared memory: written to buffer `into`).  Range mode:
+  // from the index at the first tile, else `from` (the previous tile's digits) stepped
+  // by the tile stride.
+  auto tile_digits = [&](uint64_t tile, uint8_t* into, DS from, bool first) -> DS {
     const uint64_t t = tile * 128 + row;
-    if (MODE == kTcRange) {
-      if (from == nullptr) {
+    if constexpr (RD) {
+      if (first) {
+        const uint64_t idx = R.base + t;
+        uint64_t d = 0;
+#pragma unroll
+        for (int i = 0; i < NM; ++i) d |= (uint64_t)((idx / P.stride[i]) % P.K[i]) << (8 * (NM - 1 - i));
+        return d;
+      }
+      // One add steps every digit: with each byte biased by 256 - K_i, a byte overflows
+      // exactly when its digit wraps, and the carry moves on to the next model's byte.
+      // Bytes that did not wrap then drop their bias again.
+      constexpr uint64_t ones = 0x0101010101010101ull & ((1ull << (8 * NM)) - 1);
+      const uint64_t x = from + T.dstep;
+      const uint64_t wrapped = ((x ^ from ^ T.dstep) >> 8) & ones;  // carry out of each byte
+      return (x - (~(wrapped * 0xFFull) & T.dbias)) & ((1ull << (8 * NM)) - 1);
+    } else if (MODE == kTcRange) {
+      if (first) {
         const uint64_t idx = R.base + t;
 #pragma unroll (NM > 0 ? NM : 1)
-        for (int i = 0; i < N; ++i) dg[i * 128 + row] = (uint8_t)((idx / P.stride[i]) % P.K[i]);
+        for (int i = 0; i < N; ++i) into[i * 128 + row] = (uint8_t)((idx / P.stride[i]) % P.K[i]);
       } else {  // add the tile stride to the digits, last model first
         uint32_t carry = 0;
 #pragma unroll (NM > 0 ? NM : 1)
@@ -568,26 +601,30 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
           uint32_t d = (uint32_t)from[i * 128 + row] + T.step[i] + carry;
           carry = d >= (uint32_t)P.K[i];
           if (carry) d -= (uint32_t)P.K[i];
-          dg[i * 128 + row] = (uint8_t)d;
+          into[i * 128 + row] = (uint8_t)d;
         }
       }
+      return into;
     } else {
       uint64_t idx = t < n ? L.idx[t] : 0;
       if (t < n && idx >= P.total) {
         atomicOr(P.status, kStatusBadInput);
         idx = 0;  // compute on candidate 0, discard at the end
       }
-      for (int i = 0; i < N; ++i) dg[i * 128 + row] = (uint8_t)digit_of(P, idx, i);
+      for (int i = 0; i < N; ++i) into[i * 128 + row] = (uint8_t)digit_of(P, idx, i);
+      return into;
     }
   };
-  // The aggregate state of a tile (fp32, model order) as the A1 words: bf16 hi/lo pairs.
-  auto tile_agg = [&](const uint8_t* dg) -> uint4 {
+  // The aggregate state of a tile (fp32, model order) as the A1 words: bf16 hi/lo pairs;
+  // its VRAM component (the same sum, unscaled) is the candidate's VRAM demand.
+  auto tile_agg = [&](DS dg, float& vram) -> uint4 {
     float A0 = 0.f, A1 = 0.f, A2 = 0.f;
 #pragma unroll (NM > 0 ? NM : 1)
     for (int i = 0; i < N; ++i) {
-      const float4 d = dem_s[P.off[i] + dg[i * 128 + row]];
+      const float4 d = dem_s[P.off[i] + dig(dg, i)];
       A0 += d.x; A1 += d.y; A2 += d.z;
     }
+    vram = A1;
     const float v0 = A0 * P.agg_scale[0], v1 = A1 * P.agg_scale[1], v2 = A2 * P.agg_scale[2];
     const uint32_t h0 = bf16_bits(v0), h1 = bf16_bits(v1), h2 = bf16_bits(v2);
     const uint32_t l0 = bf16_bits(v0 - __uint_as_float(h0 << 16));
@@ -595,19 +632,20 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     const uint32_t l2 = bf16_bits(v2 - __uint_as_float(h2 << 16));
     return make_uint4(h0 | (h1 << 16), h2 | (0x3F80u << 16) /* bf16 1.0 */, l0 | (l1 << 16), l2);
   };
-  // Digits of tile `tile` and its first A1 row (model m0) with the aggregate words.
-  auto load_tile = [&](uint64_t tile, uint8_t* dg, const uint8_t* from) {
-    tile_digits(tile, dg, from);
-    write_a1(m0, dg, true, tile_agg(dg));
+  // Digits of a pipeline's first tile and its first A1 row (model m0) with the aggregate words.
+  auto load_tile = [&](uint64_t tile, uint8_t* into, float& vram) -> DS {
+    const DS d = tile_digits(tile, into, DS{}, true);
+    write_a1(m0, d, true, tile_agg(d, vram));
+    return d;
   };
   // the model-i A1 row of the current tile (aggregate words already in place when AWO >= 0)
-  auto next_a1 = [&](int i, const uint8_t* dg) {
+  auto next_a1 = [&](int i, DS dg) {
     if (AWO >= 0) {
       write_a1(i, dg, false, make_uint4(0u, 0u, 0u, 0u));
     } else {  // run-time layout: the whole row, aggregate recomputed
       float A0 = 0.f, A1 = 0.f, A2 = 0.f;
       for (int j = 0; j < N; ++j) {
-        const float4 d = dem_s[P.off[j] + dg[j * 128 + row]];
+        const float4 d = dem_s[P.off[j] + dig(dg, j)];
         A0 += d.x; A1 += d.y; A2 += d.z;
       }
       const float v0 = A0 * P.agg_scale[0], v1 = A1 * P.agg_scale[1], v2 = A2 * P.agg_scale[2];
@@ -626,10 +664,13 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   const int half3 = N3 == 16 ? 8 : (T.n3 >> 1);
   float acc_J = 0.f, acc_pen = 0.f;
   bool acc_ok = true, acc_near = true;
-  auto add_model = [&](int j, const uint8_t* dg, uint64_t tile_f) {
-    const uint32_t a = tmem_ld_x1(tD3 + lane_off + (uint32_t)j);
-    const uint32_t b = tmem_ld_x1(tD3 + lane_off + (uint32_t)(half3 + j));
-    tmem_wait_ld();
+  // (the two loads are issued first; other work may run before `add_model` waits for them)
+  auto load_model = [&](int j, uint32_t& a, uint32_t& b) {
+    a = tmem_ld_x1(tD3 + lane_off + (uint32_t)j);
+    b = tmem_ld_x1(tD3 + lane_off + (uint32_t)(half3 + j));
+  };
+  auto add_model = [&](int j, uint32_t a, uint32_t b, DS dg, uint64_t tile_f) {
+    tmem_wait_ld_2(a, b);
     const float thr = tc_out(P, __uint_as_float(a) + s_b3[j][0]);
     const float lat = tc_out(P, __uint_as_float(b) + s_b3[j][1]);
     if (MODE == kTcList && L.pred) {
@@ -641,7 +682,7 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     }
     if (UT) {  // Eq. 3 utility, floors f >= tau
       float f;
-      acc_J += util_term(P, j, P.off[j] + dg[j * 128 + row], thr, &f);
+      acc_J += util_term(P, j, P.off[j] + dig(dg, j), thr, &f);
       const float tau = P.u_tau[j];
       acc_ok = acc_ok && (f >= tau);
       acc_near = acc_near && (f >= tau - 2e-2f * fmaxf(fabsf(tau), fabsf(f)));
@@ -657,7 +698,18 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   };
   // The end of a tile whose every model has been added: the VRAM bound, the earlier
   // passes' record, feasibility, the count and the top-k queue; then a fresh objective.
-  auto finish_tile = [&](uint64_t tile_f, const uint8_t* dg) {
+  // The list's k-th entry (the bar a candidate must pass to be queued) changes only in a
+  // merge; each thread keeps a copy.
+  float bar_s = -INFINITY;
+  uint64_t bar_i = kEmptyIdx;
+  auto reload_bar = [&]() {
+    if (MODE == kTcRange) {
+      const CtaTopK tk = topk();
+      bar_s = tk.ls[kcap - 1];
+      bar_i = tk.li[kcap - 1];
+    }
+  };
+  auto finish_tile = [&](uint64_t tile_f, float vram) {
     const uint64_t t = tile_f * 128 + row;
     bool valid = t < n;
     uint64_t idx;
@@ -667,9 +719,6 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
       idx = valid ? L.idx[t] : 0;
       valid = valid && idx < P.total;
     }
-    float vram = 0.f;  // the candidate's summed VRAM demand (model order, as the aggregate)
-#pragma unroll (NM > 0 ? NM : 1)
-    for (int i = 0; i < N; ++i) vram += dem_s[P.off[i] + dg[i * 128 + row]].y;
     float J = acc_J, pen = acc_pen;
     bool sla_ok = acc_ok, sla_near = acc_near;
     acc_J = 0.f;
@@ -705,7 +754,7 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     } else {
       my_count += feas ? 1u : 0u;
       const CtaTopK tk = topk();
-      const bool push = cand && precedes(J, idx, tk.ls[kcap - 1], tk.li[kcap - 1]);
+      const bool push = cand && precedes(J, idx, bar_s, bar_i);
       if (push) {
         const int pos = atomicAdd(tk.qn, 1);
         tk.qs[pos] = J;
@@ -714,7 +763,10 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
       // Candidates wait in the queue (against the list's k-th entry of the last merge)
       // until another tile's 128 might not fit; then one merge takes them all.
       named_bar(barid, 128);
-      if (*(volatile int*)tk.qn > T.qcap - 128) tc_topk_merge(tk, row, barid);
+      if (*(volatile int*)tk.qn > T.qcap - 128) {
+        tc_topk_merge(tk, row, barid);
+        reload_bar();
+      }
     }
   };
   if (issuer) {
@@ -748,10 +800,13 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     }
   } else {
     // ---- the epilogue warps ----
+    reload_bar();
     uint64_t tile = gpipe;
     int buf = 0;
+    float vram_cur = 0.f, vram_prev = 0.f, vram_nx = 0.f;  // VRAM demand of this thread's rows
+    DS dcur{}, dprev{}, dnx{};
     if (tile * 128 < n) {
-      load_tile(tile, digits, nullptr);
+      dcur = load_tile(tile, digits, vram_cur);
       signal();  // ones block and the first A1 row
     }
     // the previous tile is finished once its last layer 3 (issued at the end of that
@@ -763,24 +818,34 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     const int st_agg = m0 + 2 < m1 ? m0 + 2 : m1 - 1;
     uint4 aw_nx = make_uint4(0u, 0u, 0u, 0u);
     for (; tile * 128 < n; tile += gstride) {
-      uint8_t* dg = digits + buf * (MF_MAX_MODELS * 128);
-      uint8_t* dg_p = digits + (buf ^ 1) * (MF_MAX_MODELS * 128);
+      uint8_t* buf_nx = digits + (buf ^ 1) * (MF_MAX_MODELS * 128);  // (shared-memory digits)
       const bool has_next = (tile + gstride) * 128 < n;
+      auto stage = [&](int i) {
+        if (has_next && i == st_dig) dnx = tile_digits(tile + gstride, buf_nx, dcur, false);
+        if (has_next && i == st_agg) aw_nx = tile_agg(dnx, vram_nx);
+      };
       // Work off the critical path, while layer 2 of model i runs (or, with one hidden
       // layer, after its layer-1 epilogue): the objective terms of the model whose layer
       // 3 has landed (at the first model: the previous tile's last, and that tile's end),
-      // a stage of the next tile, the next A1 row.
+      // a stage of the next tile, the next A1 row.  The layer-3 outputs are loaded first
+      // and used last.
       auto side_work = [&](int i) {
+        uint32_t oa = 0u, ob = 0u;
         if (i > m0) {
-          add_model(i - 1, dg, tile);
-        } else if (pending) {
-          add_model(m1 - 1, dg_p, tile - gstride);
-          finish_tile(tile - gstride, dg_p);
+          load_model(i - 1, oa, ob);
+          stage(i);
+          if (i + 1 < m1) next_a1(i + 1, dcur);
+          add_model(i - 1, oa, ob, dcur, tile);
+        } else {
+          if (pending) load_model(m1 - 1, oa, ob);
+          if (i + 1 < m1) next_a1(i + 1, dcur);
+          if (pending) {  // (before the stage: with one model it overwrites these digits)
+            add_model(m1 - 1, oa, ob, dprev, tile - gstride);
+            finish_tile(tile - gstride, vram_prev);
+          }
+          stage(i);
         }
-        if (has_next && i == st_dig) tile_digits(tile + gstride, dg_p, dg);
-        if (has_next && i == st_agg) aw_nx = tile_agg(dg_p);
-        if (i + 1 < m1) next_a1(i + 1, dg);
-        else if (has_next) write_a1(m0, dg_p, true, aw_nx);
+        if (i + 1 >= m1 && has_next) write_a1(m0, dnx, true, aw_nx);
       };
 #pragma unroll (NM > 0 ? NM : 1)
       for (int i = m0; i < m1; ++i) {
@@ -810,13 +875,18 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
         signal();  // H2 stored: layer 3 of model i
       }
       pending = true;
+      dprev = dcur;
+      dcur = dnx;
+      vram_prev = vram_cur;
+      vram_cur = vram_nx;
       buf ^= 1;
     }
     if (pending) {  // the last tile's last layer 3
       await_b();
-      uint8_t* dg_last = digits + (buf ^ 1) * (MF_MAX_MODELS * 128);
-      add_model(m1 - 1, dg_last, tile - gstride);
-      finish_tile(tile - gstride, dg_last);
+      uint32_t oa, ob;
+      load_model(m1 - 1, oa, ob);
+      add_model(m1 - 1, oa, ob, dprev, tile - gstride);
+      finish_tile(tile - gstride, vram_prev);
     }
   }
   if (MODE == kTcRange && (!MP || T.pass_last) && !issuer) {  // what is still queued joins the list
@@ -1136,9 +1206,16 @@ mf_status tc_search_chunk(mf_ctx* c, const RangeArgs& a, cudaStream_t s, int* nl
   // digits of the per-tile index stride (grid x pipes x 128), modulo |Lambda|
   const uint64_t stride = ((uint64_t)c->num_sms * T.pipes * 128) % c->P.total;
   uint64_t v = stride;
+  T.dstep = 0;
+  T.dbias = 0;
   for (int i = c->P.n_models - 1; i >= 0; --i) {
     T.step[i] = (uint32_t)(v % (uint64_t)c->P.K[i]);
     v /= (uint64_t)c->P.K[i];
+    if (c->P.n_models <= 7) {
+      const int sh = 8 * (c->P.n_models - 1 - i);
+      T.dstep |= (uint64_t)(T.step[i] + 256u - (uint32_t)c->P.K[i]) << sh;
+      T.dbias |= (uint64_t)(256u - (uint32_t)c->P.K[i]) << sh;
+    }
   }
   const uint32_t smem = T.sm_total > kSmemFloor ? T.sm_total : kSmemFloor;
   TcList L{};

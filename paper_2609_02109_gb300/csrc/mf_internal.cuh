@@ -57,6 +57,9 @@ struct TcArgs {
   int32_t kcap;                       // per-pipeline list length the layout was sized for
   int32_t qcap;                       // per-pipeline candidate queue (128 or 512, a power of two)
   uint32_t step[MF_MAX_MODELS];       // mixed-radix digits of the per-tile index stride (range mode)
+  // the same stride for digits packed one per byte (model N - 1 in the lowest byte):
+  // byte of model i = step[i] + 256 - K_i, and the bias bytes 256 - K_i
+  uint64_t dstep, dbias;
   // models whose weights do not fit shared memory together run in passes of consecutive
   // models [pass_m[p], pass_m[p + 1]); each pass's image is staged on its own
   int32_t npasses;
