@@ -175,23 +175,8 @@ class Context:
     def __init__(self, prob: dict, device: int | None = None, precision: str | None = None):
         self.device = torch.cuda.current_device() if device is None else int(device)
         prec = precision or prob.get("precision", "fp32")
-        self._keep = {
-            "n_options": np.ascontiguousarray(prob["n_options"], dtype=np.int32),
-            "local_feats": _f32(prob["local_feats"]), "demand": _f32(prob["demand"]),
-            "weights": _f32(prob["weights"]),
-            "agg_scale": None if prob.get("agg_scale") is None else _f32(prob["agg_scale"]),
-            "sla": _f32(prob["sla"]), "obj_w": _f32(prob["obj_w"]),
-        }
-        k = self._keep
-        ptr = lambda a: None if a is None else a.ctypes.data  # noqa: E731
-        self.n_models = int(k["n_options"].size)
-        p = _Problem(self.n_models, ptr(k["n_options"]), int(prob["d_local"]), int(prob["hidden1"]),
-                     int(prob["hidden2"]), ptr(k["local_feats"]), ptr(k["demand"]), ptr(k["weights"]),
-                     ptr(k["agg_scale"]), ptr(k["sla"]), ptr(k["obj_w"]),
-                     float(prob["vram_cap"]), float(prob.get("soft_penalty", 0.0)),
-                     1 if prob.get("out_act", "identity") == "sigmoid" else 0,
-                     1 if prob.get("objective", "weighted_thr") == "soft_lat" else 0,
-                     MF_BF16 if prec == "bf16" else MF_FP32, self.device)
+        p, self._keep = _problem_struct(prob, self.device, prec)
+        self.n_models = int(p.n_models)
         h = C.c_void_p()
         with torch.cuda.device(self.device):
             _check(_lib.mf_create(C.byref(p), C.byref(h)), "mf_create")
