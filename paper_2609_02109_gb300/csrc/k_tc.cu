@@ -92,10 +92,6 @@ __device__ __forceinline__ void named_bar(int id, int nthreads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
 
-__device__ __forceinline__ void named_arrive(int id, int nthreads) {
-  asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
-}
-
 // OR of `pred` over the threads of a named barrier (also a barrier).
 __device__ __forceinline__ bool named_bar_or(int id, int nthreads, bool pred) {
   uint32_t r;
@@ -467,9 +463,12 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   uint64_t* barA = &bars[1 + 2 * pipe];  // layers 1 and 2 completed (alternating)
   uint64_t* barB = &bars[2 + 2 * pipe];  // layer 3 completed
   uint32_t phA = 0, phB = 0;
-  // epilogue -> issuer hand-offs alternate between two named barriers per pipeline (the
-  // epilogue warps arrive, the issuing warp syncs; the epilogue warps never run two
-  // hand-offs ahead); the pipeline's top-k uses a third among its epilogue warps
+  // epilogue -> issuer hand-offs alternate between two named barriers per pipeline, each
+  // a full rendezvous of the 160 threads: the epilogue warps cannot run ahead of the
+  // issuing warp even where their mbarrier waits return early (after a wait gave up),
+  // which with arrive-only hand-offs could complete a barrier without the issuing warp
+  // and leave it waiting at the next one; the pipeline's top-k uses a third barrier
+  // among its epilogue warps
   const int sig0 = 1 + 2 * pipe, barid = 1 + 2 * npipes + pipe;
   const uint32_t id1 = idesc_bf16(T.h1), id2 = idesc_bf16(T.h2), id3 = idesc_bf16(T.n3);
   const int s1 = T.k1 / 16, s2 = T.h1 / 16 + 1, s3 = T.hl / 16;
@@ -521,7 +520,7 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   auto signal = [&]() {
     tmem_wait_st();
     tc_fence_before();
-    named_arrive(sig0 + (int)(ksig & 1u), 160);
+    named_bar(sig0 + (int)(ksig & 1u), 160);
     ++ksig;
   };
   // issuing warp: the epilogue warps' next hand-off
