@@ -140,41 +140,68 @@ k_fc_local(const Params P, const FcLayout L, const FcConst C) {
 
 // ---------------------------------------------------------------------------
 // Table-lookup scan.  Each thread walks its own contiguous slice of the range, so from
-// one candidate to the next only the last model's option advances (the partial sum
-// over the other models is reused until a carry).  J is summed in model order either
-// way.  Per-CTA running top-k as in the fp32 scorer: every RUN candidates of each
-// thread, one merge check with a queue of one entry per candidate of the step.
+// one candidate to the next only the last model's option advances: the partial sum over
+// the other models is reused until a carry, and a carry that stops at model N - 2 (all
+// but one in K_{N-2}) costs one lookup.  J is summed in model order either way.
+// Running top-k: a thread queues a candidate only if it beats the list's k-th entry
+// (held in registers), at most kFcBudget between two merge checks (a thread that runs
+// out stops until the merge); a merge check follows every cycle of the last model's
+// options, at least kFcMinRun candidates (kFcMinRunLong in slices long enough that the
+// list settles early).  WL (k <= kFcWarpK): each warp keeps its own list and queue and
+// merges with warp barriers only, the CTA's list taking the warps' lists at the end;
+// otherwise one list per CTA, the merge check a CTA barrier.
 // ---------------------------------------------------------------------------
 constexpr int kFcThreads = 512;
-// Runs of 16 halve the per-step barriers of long scans; runs of 8 keep the first step's
-// queue (every feasible candidate of the step, sorted before the merge) short.
-constexpr int kFcRunLong = 16, kFcRunShort = 8;
-constexpr uint64_t kFcLongScan = 1ull << 29;
+constexpr int kFcBudget = 8;   // the queue: kFcThreads x kFcBudget entries
+constexpr int kFcMinRun = 16, kFcMinRunLong = 64;
+constexpr int kFcWarpK = 64, kFcWarps = kFcThreads / 32;
+constexpr int kFcWarpQ = 32 * kFcBudget;              // a warp's queue
+constexpr int kFcEndQ = kFcWarps * kFcWarpK;          // the warps' lists, merged at the end (a power of two)
+constexpr uint64_t kFcLongSlice = 8192;
 
 struct FcScan {
   const float2* tab;
 };
 
-template <int RUN, int NMAX>
+// Shared-memory bytes of k_fc_scan<.., WL> after the table.
+__host__ __device__ inline size_t fc_scan_list_bytes(int k, bool wl) {
+  const size_t e = sizeof(uint64_t) + sizeof(float);
+  if (!wl) return e * (2 * (size_t)k + kFcThreads * kFcBudget) + 16;
+  return e * (2 * (size_t)k + kFcEndQ) + 16 + kFcWarps * (e * (2 * (size_t)k + kFcWarpQ) + 16);
+}
+
+template <int NMAX, bool WL>
 __global__ void __launch_bounds__(kFcThreads, 1)
 k_fc_scan(const Params P, const FcScan S, const RangeArgs R) {
-  constexpr int kFcRun = RUN;  // NMAX: a bound on N for the unrolled per-model loops
+  // NMAX: a bound on N for the unrolled per-model loops
   extern __shared__ __align__(16) unsigned char sm[];
   const int N = P.n_models;
   const int sumK = pick(P.off, N - 1) + pick(P.K, N - 1);
-  constexpr int QCAP = kFcThreads * kFcRun;
+  constexpr int QCAP = WL ? kFcEndQ : kFcThreads * kFcBudget;
   float2* tab = reinterpret_cast<float2*>(sm);
   unsigned char* q = sm + (((size_t)sumK * sizeof(float2) + 15) & ~(size_t)15);
-  const int tid = threadIdx.x;
-  CtaTopK tk;
-  tk.li = reinterpret_cast<uint64_t*>(q); q += sizeof(uint64_t) * R.k;
-  tk.ni = reinterpret_cast<uint64_t*>(q); q += sizeof(uint64_t) * R.k;
-  tk.qi = reinterpret_cast<uint64_t*>(q); q += sizeof(uint64_t) * QCAP;
-  tk.ls = reinterpret_cast<float*>(q); q += sizeof(float) * R.k;
-  tk.ns = reinterpret_cast<float*>(q); q += sizeof(float) * R.k;
-  tk.qs = reinterpret_cast<float*>(q); q += sizeof(float) * QCAP;
-  tk.qn = reinterpret_cast<int*>(q);
-  tk.k = R.k;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  // one list + queue block: li, ni [k], qi [qcap], ls, ns [k], qs [qcap], qn
+  auto carve = [&](CtaTopK& t, int qcap) {
+    t.li = reinterpret_cast<uint64_t*>(q); q += sizeof(uint64_t) * R.k;
+    t.ni = reinterpret_cast<uint64_t*>(q); q += sizeof(uint64_t) * R.k;
+    t.qi = reinterpret_cast<uint64_t*>(q); q += sizeof(uint64_t) * qcap;
+    t.ls = reinterpret_cast<float*>(q); q += sizeof(float) * R.k;
+    t.ns = reinterpret_cast<float*>(q); q += sizeof(float) * R.k;
+    t.qs = reinterpret_cast<float*>(q); q += sizeof(float) * qcap;
+    t.qn = reinterpret_cast<int*>(q); q += 16;
+    t.k = R.k;
+  };
+  CtaTopK tk, wt;  // the CTA's list; this warp's (WL), else the CTA's again
+  carve(tk, QCAP);
+  if (WL) {  // the warps' blocks follow the CTA's, in warp order
+    q += (size_t)warp * ((sizeof(uint64_t) + sizeof(float)) * (2 * (size_t)R.k + kFcWarpQ) + 16);
+    carve(wt, kFcWarpQ);
+    for (int e = lane; e < R.k; e += 32) { wt.ls[e] = -INFINITY; wt.li[e] = kEmptyIdx; }
+    if (lane == 0) *wt.qn = 0;
+  } else {
+    wt = tk;
+  }
   // an option below its floor (utility -inf, or NaN) carries VRAM +inf here, so one
   // compare against the cap decides feasibility
   for (int e = tid; e < sumK; e += blockDim.x) {
@@ -188,93 +215,157 @@ k_fc_scan(const Params P, const FcScan S, const RangeArgs R) {
     tk.li[e] = R.first ? kEmptyIdx : R.lists_i[gl + e];
   }
   if (tid == 0) *tk.qn = 0;
-  // Thread g of the grid scans the contiguous slice [g S, (g + 1) S) of the range, RUN
-  // candidates between two merge checks; its option rows, the prefix sum over models
-  // 0..N-2 and the last model's row carry from run to run.  S = ceil(len / threads); in
-  // long scans rounded up to a multiple of the last model's option count, so all lanes
-  // of a warp reach a carry at the same candidate (no divergence in the scan loop),
-  // while short scans keep slices short (a small first merge, spread over more CTAs).
+  // Thread g of the grid scans the contiguous slice [g S, (g + 1) S) of the range.
+  // S = ceil(len / threads); in long scans rounded up to a multiple of the last model's
+  // option count, so all lanes of a warp run the same cycles of the last model's options
+  // (the same table entries, no divergence), while short scans keep slices short (a small
+  // first merge, spread over more CTAs).
   const uint64_t nthreads = (uint64_t)gridDim.x * blockDim.x;
-  const uint64_t klast = (uint64_t)pick(P.K, N - 1);
+  const int last = N - 1;
+  const int off_last = pick(P.off, last);
+  const int klast = pick(P.K, last);
   const uint64_t slice0 = (R.len + nthreads - 1) / nthreads;
-  const uint64_t slice = slice0 >= 4 * klast ? (slice0 + klast - 1) / klast * klast : slice0;
+  const uint64_t slice = slice0 >= 4 * (uint64_t)klast ? (slice0 + klast - 1) / klast * klast : slice0;
   const uint64_t s0 = ((uint64_t)blockIdx.x * blockDim.x + tid) * slice;
   const uint64_t s1 = s0 + slice < R.len ? s0 + slice : R.len;
-  int row[NMAX];
+  int row[NMAX];  // option rows of models 0 .. N - 2
+  int o;          // the last model's option
   {
     const uint64_t idx0 = R.base + (s0 < R.len ? s0 : 0);
 #pragma unroll
     for (int i = 0; i < NMAX; ++i)
-      if (i < N) row[i] = P.off[i] + (int)((idx0 / P.stride[i]) % (uint64_t)P.K[i]);
+      if (i < last) row[i] = P.off[i] + (int)((idx0 / P.stride[i]) % (uint64_t)P.K[i]);
+    o = (int)((idx0 / pick(P.stride, last)) % (uint64_t)klast);
   }
   __syncthreads();
   float thr_s = tk.ls[R.k - 1];
   uint64_t thr_i = tk.li[R.k - 1];
   const float cap = P.vram_cap;
-  const int last = N - 1;
-  const int off_last = pick(P.off, last);
-  const int end_last = off_last + pick(P.K, last);
+  // prefix sums in model order: p2 over models 0 .. N - 3, p over 0 .. N - 2; rp is
+  // model N - 2's option row (the one a carry usually stops at), endp its end
+  float pJ2 = 0.f, pV2 = 0.f, pJ = 0.f, pV = 0.f;
+  int rp = 0, endp = 0;
+  auto prefix = [&]() {
+    pJ2 = 0.f;
+    pV2 = 0.f;
+#pragma unroll
+    for (int i = 0; i < NMAX; ++i)
+      if (i < last - 1) { const float2 e = tab[row[i]]; pJ2 += e.x; pV2 += e.y; }
+    pJ = pJ2;
+    pV = pV2;
+    if (last >= 1) {
+#pragma unroll
+      for (int i = 0; i < NMAX; ++i)
+        if (i == last - 1) rp = row[i];
+      const float2 e = tab[rp];
+      pJ += e.x;
+      pV += e.y;
+    }
+  };
+  if (last >= 1) endp = pick(P.off, last - 1) + pick(P.K, last - 1);
+  prefix();
+  const float thr0_s = thr_s;  // (WL: the bar until the warp's own list is full)
+  const uint64_t thr0_i = thr_i;
+  // the last model's option wrapped: the next option of the models before it
+  auto carry = [&]() {
+    if (++rp < endp) {
+      const float2 e = tab[rp];
+      pJ = pJ2 + e.x;
+      pV = pV2 + e.y;
+      return;
+    }
+    bool c = true;  // model N - 2 wrapped as well
+#pragma unroll
+    for (int i = NMAX - 1; i >= 0; --i)
+      if (i < last && c) {
+        const int off = P.off[i];
+        int d = (i == last - 1 ? rp : row[i] + 1) - off;
+        c = d == P.K[i];
+        if (c) d = 0;
+        row[i] = off + d;
+      }
+    prefix();
+  };
+  const float2* tl = tab + off_last;
+  const int minrun = slice >= kFcLongSlice ? kFcMinRunLong : kFcMinRun;
+  uint64_t t = s0;  // this thread's next candidate (offset in the range)
+  bool done = t >= s1;
   unsigned int my_count = 0;
-  float pJ = 0.f, pV = 0.f;
-#pragma unroll
-  for (int i = 0; i < NMAX; ++i)
-    if (i < last) { const float2 e = tab[row[i]]; pJ += e.x; pV += e.y; }
-  int rl = row[0];
-#pragma unroll
-  for (int i = 1; i < NMAX; ++i)
-    if (i == last) rl = row[i];
-  const uint64_t nruns = (slice + kFcRun - 1) / kFcRun;  // the same for every thread
-  for (uint64_t r = 0; r < nruns; ++r) {
-    bool any = false;
-    const uint64_t t1 = s0 + r * kFcRun;
-    const int nv = t1 >= s1 ? 0 : (s1 - t1 >= (uint64_t)kFcRun ? kFcRun : (int)(s1 - t1));
-    // the run in segments between carries of the last model's option: a segment is a
-    // plain loop (one lookup, two adds, one compare per candidate); the carry into the
-    // prefix runs between segments
-    int u0 = 0;
-    while (u0 < nv) {
-      const int seg = min(nv - u0, end_last - rl);
-      for (int u = u0; u < u0 + seg; ++u, ++rl) {
-        const float2 e = tab[rl];
-        const float J = pJ + e.x, V = pV + e.y;
-        const bool feas = V <= cap;  // NaN compares false
+  for (;;) {
+    int pushed = 0, ran = 0;
+    while (!done && ran < minrun) {
+      const int n_here = s1 - t < (uint64_t)(klast - o) ? (int)(s1 - t) : klast - o;
+      const float2* e0 = tl + o;
+      // fast pass: the count, and whether any candidate might enter the list
+      bool hit = false;
+      const float2 pjv = make_float2(pJ, pV);
+#pragma unroll 8
+      for (int u = 0; u < n_here; ++u) {
+        const float2 jv = __fadd2_rn(pjv, e0[u]);  // (J, V) = (pJ + x, pV + y), one paired add
+        const bool feas = jv.y <= cap;  // NaN compares false
         my_count += feas ? 1u : 0u;
-        if (feas && J >= thr_s) {  // rare once the list is full; the index only then
-          const uint64_t idx = R.base + t1 + u;
-          if (precedes(J, idx, thr_s, thr_i)) {
-            const int pos = atomicAdd(tk.qn, 1);
-            tk.qs[pos] = J;
-            tk.qi[pos] = idx;
-            any = true;
+        hit |= feas & (jv.x >= thr_s);
+      }
+      int u = n_here;
+      if (hit) {  // rare once the list is full: queue what beats its k-th entry
+        for (u = 0; u < n_here; ++u) {
+          const float2 e = e0[u];
+          const float J = pJ + e.x, V = pV + e.y;
+          if (V <= cap && J >= thr_s) {
+            const uint64_t idx = R.base + t + u;
+            if (precedes(J, idx, thr_s, thr_i)) {
+              if (pushed == kFcBudget) break;  // this candidate and the rest wait for the merge
+              const int pos = atomicAdd(wt.qn, 1);
+              wt.qs[pos] = J;
+              wt.qi[pos] = idx;
+              ++pushed;
+            }
           }
         }
+        for (int w = u; w < n_here; ++w) my_count -= (pV + e0[w].y <= cap) ? 1u : 0u;  // counted again later
       }
-      u0 += seg;
-      if (rl == end_last) {  // carry into the prefix
-        rl = off_last;
-        bool carry = true;
-#pragma unroll
-        for (int i = NMAX - 1; i >= 0; --i)
-          if (i < last && carry) {
-            const int off = P.off[i];
-            int d = row[i] - off + 1;
-            carry = d == P.K[i];
-            if (carry) d = 0;
-            row[i] = off + d;
-          }
-        pJ = 0.f;
-        pV = 0.f;
-#pragma unroll
-        for (int i = 0; i < NMAX; ++i)
-          if (i < last) { const float2 e2 = tab[row[i]]; pJ += e2.x; pV += e2.y; }
-      }
+      t += u;
+      o += u;
+      ran += u;
+      if (t >= s1) done = true;
+      else if (o == klast) { o = 0; carry(); }
+      if (u < n_here) break;
     }
-    if (__syncthreads_or(any)) {  // block-uniform
-      // a queue that fills a whole run (the first runs of a search) is sorted first
-      if (*tk.qn > 256) topk_merge_sorted(tk, tid, blockDim.x, [] __device__() { __syncthreads(); });
+    if (WL) {
+      const bool more = __any_sync(0xffffffffu, !done);
+      if (__any_sync(0xffffffffu, pushed > 0)) {
+        __syncwarp();
+        if (*(volatile int*)wt.qn > 32) topk_merge_sorted(wt, lane, 32, [] __device__() { __syncwarp(); });
+        else topk_merge(wt, lane, 32, [] __device__() { __syncwarp(); });
+        const bool full = wt.li[R.k - 1] != kEmptyIdx;  // (its entries all beat the CTA's bar)
+        thr_s = full ? wt.ls[R.k - 1] : thr0_s;
+        thr_i = full ? wt.li[R.k - 1] : thr0_i;
+      }
+      if (!more) break;
+    } else {
+      const bool more = __syncthreads_or(!done);
+      if (*(volatile int*)tk.qn > 0) {  // (read by every thread after the barrier: uniform)
+        // a long queue (the first merges of a search) is sorted first
+        if (*(volatile int*)tk.qn > 256) topk_merge_sorted(tk, tid, blockDim.x, [] __device__() { __syncthreads(); });
+        else topk_merge(tk, tid, blockDim.x, [] __device__() { __syncthreads(); });
+        thr_s = tk.ls[R.k - 1];
+        thr_i = tk.li[R.k - 1];
+      }
+      if (!more) break;
+    }
+  }
+  if (WL) {  // the warps' lists join the CTA's
+    __syncthreads();
+    for (int e = lane; e < R.k; e += 32)
+      if (wt.li[e] != kEmptyIdx) {
+        const int pos = atomicAdd(tk.qn, 1);
+        tk.qs[pos] = wt.ls[e];
+        tk.qi[pos] = wt.li[e];
+      }
+    __syncthreads();
+    if (*(volatile int*)tk.qn > 0) {
+      if (*(volatile int*)tk.qn > 256) topk_merge_sorted(tk, tid, blockDim.x, [] __device__() { __syncthreads(); });
       else topk_merge(tk, tid, blockDim.x, [] __device__() { __syncthreads(); });
-      thr_s = tk.ls[R.k - 1];
-      thr_i = tk.li[R.k - 1];
     }
   }
   for (int e = tid; e < R.k; e += blockDim.x) {
@@ -401,8 +492,9 @@ static void radix_digits(const Params& P, uint64_t v, uint32_t* step) {
 // GA of k_ga.cu with two more: crossover applied with probability crossover_p (draw
 // kGaCrossDo, else the first parent is copied) and repair of an infeasible individual
 // by rejection sampling from the uniform distribution over Lambda (draws kGaRepair,
-// j = a * N + i, at most 256 / N attempts, the first feasible one kept).  A warp's
-// repairs share its lanes (see repair_warp).
+// j = a * N + i, at most 256 / N attempts, the first feasible one kept).  The block has
+// 1024 threads whatever the population, and a generation's repairs share all of them
+// (see repair).
 // ---------------------------------------------------------------------------
 struct FcGaArgs {
   const float2* tab;
@@ -428,6 +520,8 @@ k_fc_ga(const Params P, const FcGaArgs A) {
   extern __shared__ __align__(16) unsigned char sm[];
   __shared__ float sval[32];
   __shared__ int sidx[32];
+  __shared__ int s_wcnt[32];
+  __shared__ int s_pend[1024];
   const int N = P.n_models, pop = A.pop;
   const int sumK = pick(P.off, N - 1) + pick(P.K, N - 1);
   float2* tab = reinterpret_cast<float2*>(sm);
@@ -440,27 +534,33 @@ k_fc_ga(const Params P, const FcGaArgs A) {
   __syncthreads();
   const uint64_t sd = A.seed;
   const int attempts = 256 / N;
-  // Repair of the warp's infeasible children (need): the m of them (rounded up to a
-  // power of two) each get a group of 32 / m lanes, which tries the child's attempts
-  // 32 / m at a time; the lowest feasible attempt of a group's first successful round is
-  // the sequential search's result.  The winning lane writes the child's genes and
-  // fitness over the unrepaired ones already in shared memory.  With 32 pending
-  // children this is the sequential search on every lane.
-  const int lane = c & 31;
-  auto repair_warp = [&](uint32_t G, bool need, uint8_t* genes, float* fit) {
-    __syncwarp();
-    const unsigned pend = __ballot_sync(0xffffffffu, need);
-    if (!pend) return;
-    const int cnt = __popc(pend);
+  // Repair of the generation's infeasible children (need): the cnt of them, in ascending
+  // order, each get a group of gs lanes of one warp (gs a power of two, as many lanes as
+  // the block has for cnt rounded up to a power of two, at most 32), which tries the
+  // child's attempts gs at a time; the lowest feasible attempt of a group's first
+  // successful round is the sequential search's result.  The winning lane writes the
+  // child's genes and fitness over the unrepaired ones already in shared memory.
+  const int lane = c & 31, warp = c >> 5, nwarps = (int)(blockDim.x >> 5);
+  auto repair = [&](uint32_t G, bool need, uint8_t* genes, float* fit) {
+    const unsigned bal = __ballot_sync(0xffffffffu, need);
+    if (lane == 0) s_wcnt[warp] = __popc(bal);
+    __syncthreads();
+    int before = 0, cnt = 0;
+    for (int w = 0; w < (pop + 31) / 32; ++w) {  // (only the population's warps breed)
+      const int v = s_wcnt[w];
+      before += w < warp ? v : 0;
+      cnt += v;
+    }
+    if (need) s_pend[before + __popc(bal & ((1u << lane) - 1u))] = c;
+    __syncthreads();
+    if (cnt == 0) return;  // (uniform)
     int m = 1;
     while (m < cnt) m <<= 1;
-    const int gs = 32 / m, grp = lane / gs, lig = lane % gs;
-    int child = -1;
-    if (grp < cnt) {
-      unsigned x = pend;
-      for (int q = 0; q < grp; ++q) x &= x - 1;
-      child = (c & ~31) + __ffs(x) - 1;
-    }
+    int gs = nwarps * 32 / m;
+    gs = gs > 32 ? 32 : (gs < 1 ? 1 : gs);
+    const int grp = lane / gs, lig = lane % gs;
+    const int gid = warp * (32 / gs) + grp;
+    const int child = gid < cnt ? s_pend[gid] : -1;
     const unsigned gmask = gs == 32 ? 0xffffffffu : ((1u << gs) - 1u) << (grp * gs);
     bool done = child < 0;
     for (int a0 = 0; a0 < attempts; a0 += gs) {
@@ -493,7 +593,6 @@ k_fc_ga(const Params P, const FcGaArgs A) {
         done = true;
       }
     }
-    __syncwarp();
   };
   bool need = false;
   if (c < pop) {  // initial population: uniform over Lambda, repaired
@@ -503,7 +602,7 @@ k_fc_ga(const Params P, const FcGaArgs A) {
     fit0[c] = J;
     need = A.repair && J == -INFINITY;
   }
-  repair_warp(0u, need, g0, fit0);
+  repair(0u, need, g0, fit0);
   __syncthreads();
   uint8_t* gc = g0;
   uint8_t* gn = g1;
@@ -545,7 +644,7 @@ k_fc_ga(const Params P, const FcGaArgs A) {
       fn[c] = J;
       need = A.repair && J == -INFINITY;
     }
-    repair_warp(G, need, gn, fn);
+    repair(G, need, gn, fn);
     __syncthreads();
     uint8_t* tg = gc; gc = gn; gn = tg;
     float* tf = fc_; fc_ = fn; fn = tf;
@@ -562,17 +661,16 @@ mf_status fc_search_chunk(mf_ctx* c, const RangeArgs& a, cudaStream_t s) {
   fc_bytes(c->sumK, c->P.n_models, &L, (char*)c->d_fc);
   FcScan S{};
   S.tab = L.tab;
-  const int run = a.len >= kFcLongScan ? kFcRunLong : kFcRunShort;
-  const size_t smem = (((size_t)c->sumK * sizeof(float2) + 15) & ~(size_t)15) +
-                      (sizeof(uint64_t) + sizeof(float)) * (2 * (size_t)a.k + kFcThreads * run) + 16;
+  const bool wl = a.k <= kFcWarpK;  // per-warp lists
+  const size_t smem = (((size_t)c->sumK * sizeof(float2) + 15) & ~(size_t)15) + fc_scan_list_bytes(a.k, wl);
   if (smem > 227 * 1024) {
     set_error("fixed-context search: top-k lists do not fit shared memory; use a smaller k");
     return MF_EUNSUPPORTED;
   }
   using ScanFn = void (*)(const Params, const FcScan, const RangeArgs);
-  const bool small_n = c->P.n_models <= 8;
-  const ScanFn fn = run == kFcRunLong ? (small_n ? k_fc_scan<kFcRunLong, 8> : k_fc_scan<kFcRunLong, MF_MAX_MODELS>)
-                                      : (small_n ? k_fc_scan<kFcRunShort, 8> : k_fc_scan<kFcRunShort, MF_MAX_MODELS>);
+  const bool n8 = c->P.n_models <= 8;
+  const ScanFn fn = wl ? (n8 ? k_fc_scan<8, true> : k_fc_scan<MF_MAX_MODELS, true>)
+                       : (n8 ? k_fc_scan<8, false> : k_fc_scan<MF_MAX_MODELS, false>);
   MF_CUDA(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
   fn<<<fc_grid(c), kFcThreads, smem, s>>>(c->P, S, a);
   MF_CUDA(cudaGetLastError());
@@ -729,7 +827,7 @@ mf_status mf_fc_ga_run(mf_ctx* ctx, const mf_fc_ga_params* g, uint64_t seed, int
   A.out_genome = (int32_t*)ctx->d_scratch;
   A.out_fit = (float*)((int32_t*)ctx->d_scratch + 16);
   const size_t smem = sizeof(float2) * ctx->sumK + sizeof(float) * 2 * g->pop + (size_t)2 * g->pop * N;
-  const int threads = (g->pop + 31) / 32 * 32;
+  const int threads = 1024;  // (the repairs use every warp)
   MF_CUDA(cudaFuncSetAttribute(k_fc_ga, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
   k_fc_ga<<<1, threads, smem, s>>>(ctx->P, A);
   MF_CUDA(cudaGetLastError());

@@ -182,7 +182,9 @@ __device__ __forceinline__ int block_argmax(const float* __restrict__ fit, int n
     const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
     if (oi != 0x7fffffff && (bi == 0x7fffffff || ob > best || (ob == best && oi < bi))) { best = ob; bi = oi; }
   }
-  const int w = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+  const int w = threadIdx.x >> 5;
+  const int nwb = (blockDim.x + 31) >> 5, nwn = (n + 31) >> 5;
+  const int nw = nwn < nwb ? nwn : nwb;  // warps holding entries (the rest found none)
   if ((threadIdx.x & 31) == 0) { sval[w] = best; sidx[w] = bi; }
   __syncthreads();
   if (threadIdx.x == 0) {

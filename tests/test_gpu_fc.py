@@ -112,7 +112,7 @@ def test_fc_table_matches_oracle(mf, oracle_mod, name):
 
 
 @pytest.mark.parametrize("name", list(CASES))
-@pytest.mark.parametrize("k", [1, 8, 32])
+@pytest.mark.parametrize("k", [1, 8, 32, 100])  # (up to 64: per-warp lists; 100: one list per CTA)
 def test_fc_search_matches_oracle(mf, oracle_mod, name, k):
     prob, fc = CASES[name]
     o = oracle_mod.Oracle(prob)
@@ -164,8 +164,8 @@ def test_fc_full_size_separable_closed_form(mf, oracle_mod, which, seed, chunk):
     """At full size (24^6 and 16^8 candidates) the VRAM cap of 180 GB never binds, so
     the feasible count is the product of the per-model floor-feasible option counts
     and the best configuration takes each model's best feasible option (from the
-    oracle's per-option table).  Chunks of 2^26 scan in runs of 8 candidates per
-    thread, chunks of 2^30 in runs of 16."""
+    oracle's per-option table).  Chunks of 2^26 and 2^30 give the scan's threads short
+    and long slices."""
     prob = W.large(precision="fp32") if which == "large" else W.stress(precision="fp32")
     fc = W.fc_scenario(prob, seed)
     o = oracle_mod.Oracle(prob)
@@ -256,3 +256,19 @@ def test_paper_ga_decisions_on_the_paper_landscape(mf, oracle_mod):
                 Jo, feas = o.fc_score_digits(fc, g)
                 assert feas and abs(J - Jo) <= 1e-5 * max(1.0, abs(Jo))
                 assert Jo >= ts[0] - 0.005 * abs(ts[0])
+
+
+@pytest.mark.parametrize("chunk", [1 << 22, 1 << 30])
+def test_fc_search_warp_lists_equal_cta_list(mf, chunk):
+    """The scan keeps per-warp lists for k <= 64 and one list per CTA above: on the
+    large space (24^6) the first 64 entries of a top-128 search (CTA list) equal a
+    top-64 search (warp lists), and the counts agree."""
+    prob = W.large(precision="fp32")
+    fc = W.fc_scenario(prob, 3)
+    with mf.Context(prob) as ctx:
+        ctx.fc_set(fc)
+        a = ctx.fc_search(64, chunk=chunk)
+        b = ctx.fc_search(128, chunk=chunk)
+    assert a["count"] == b["count"]
+    np.testing.assert_array_equal(np.asarray(a["topk_idx"]), np.asarray(b["topk_idx"])[:64])
+    np.testing.assert_array_equal(np.asarray(a["topk_score"]), np.asarray(b["topk_score"])[:64])
