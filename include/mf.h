@@ -53,7 +53,13 @@ typedef enum {
   MF_EDEVICE = 6        /* the device reported an invalid input (e.g. an index >= |Lambda|) */
 } mf_status;
 
-typedef enum { MF_FP32 = 0, MF_BF16 = 1 } mf_precision;
+/* MF_FP32: fp32 results (scores within 1e-5 of the fp64 definition).  For the
+ * d_L 8, 12 -> 64 -> 64 -> 2 predictor shape (up to 8 models) the scoring runs on the
+ * tensor cores with every operand split into two tf32 parts (hi.hi + hi.lo + lo.hi,
+ * about 22 bits per product, fp32 accumulation); other shapes run on the CUDA cores.
+ * MF_FP32_SIMT: the same results on the CUDA cores for every shape.
+ * MF_BF16: bf16 tensor-core scoring, search results re-scored in fp32. */
+typedef enum { MF_FP32 = 0, MF_BF16 = 1, MF_FP32_SIMT = 2 } mf_precision;
 /* MF_OBJ_UTILITY (Eq. 3 utility with floors) is set with mf_set_utility only. */
 typedef enum { MF_OBJ_WEIGHTED_THR = 0, MF_OBJ_SOFT_LAT = 1, MF_OBJ_UTILITY = 2 } mf_objective;
 typedef enum { MF_ACT_IDENTITY = 0, MF_ACT_SIGMOID = 1 } mf_out_act;
@@ -123,6 +129,8 @@ typedef struct {
                                   launch of the last search */
   float total_ms_last;         /* device time of the whole last search (scoring, merge,
                                   re-scoring, result copy) */
+  int32_t scoring_path;        /* the context's scoring kernels: 0 fp32 on the CUDA cores,
+                                  1 bf16 tensor cores, 2 fp32 tensor cores (3-term tf32) */
 } mf_stats;
 
 /* Name of a status code (static string). */

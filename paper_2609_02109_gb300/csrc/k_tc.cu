@@ -116,6 +116,11 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int n) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
 }
 
+// Instruction descriptor of kind::tf32: tf32 A and B (K-major), fp32 D, M = 128.
+__host__ __device__ constexpr uint32_t idesc_tf32(int n) {
+  return (1u << 4) | (2u << 7) | (2u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
+}
+
 // D[tmem] (+)= A[tmem] . B[smem]^T, one 128 x n x 16 MMA.
 __device__ __forceinline__ void mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
                                        uint32_t accumulate) {
@@ -141,6 +146,13 @@ __device__ __forceinline__ uint32_t relu_bf16x2(uint32_t lo, uint32_t hi) {
 
 __device__ __forceinline__ uint32_t bf16_bits(float v) {
   return (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v));
+}
+
+// v rounded to tf32 (nearest, ties away from zero): its fp32 bits, low 13 bits zero.
+__device__ __forceinline__ uint32_t tf32_bits(float v) {
+  uint32_t d;
+  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(d) : "f"(v));
+  return d;
 }
 
 __device__ __forceinline__ uint32_t tmem_ld_x1(uint32_t taddr) {
@@ -170,6 +182,13 @@ __device__ __forceinline__ void tmem_st_x4(uint32_t taddr, const uint32_t (&v)[4
 __device__ __forceinline__ void tmem_st_x8(uint32_t taddr, const uint32_t (&v)[8]) {
   asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};"
                :: "r"(taddr), "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7])
+               : "memory");
+}
+
+__device__ __forceinline__ void tmem_st_x32(uint32_t taddr, const uint32_t (&v)[32]) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};"
+               :: "r"(taddr), "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15]),
+                  "r"(v[16]), "r"(v[17]), "r"(v[18]), "r"(v[19]), "r"(v[20]), "r"(v[21]), "r"(v[22]), "r"(v[23]), "r"(v[24]), "r"(v[25]), "r"(v[26]), "r"(v[27]), "r"(v[28]), "r"(v[29]), "r"(v[30]), "r"(v[31])
                : "memory");
 }
 
@@ -278,6 +297,31 @@ __device__ __forceinline__ void mma_commit_warp(uint64_t* bar) {
       : "memory");
 }
 
+// The same for kind::tf32 (one 128 x n x 8 MMA).
+__device__ __forceinline__ void mma_ts_warp_tf32(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                                                 uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p, e;\n setp.ne.b32 p, %4, 0;\n elect.sync _|e, 0xffffffff;\n"
+      " @e tcgen05.mma.cta_group::1.kind::tf32 [%0], [%1], %2, %3, p;\n}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// The three products of the exact fp32 variant, A = a_hi + a_lo and B = b_hi + b_lo in
+// tf32 parts: KH K-steps of A_hi B_hi, then KX of A_hi B_lo and of A_lo B_hi (A_lo B_lo,
+// about 2^-22 of the product, is left out).  A K-step is 8 columns of A and 256 bytes
+// of B.
+template <int KH, int KX>
+__device__ __forceinline__ void mma_tf3(uint32_t d, uint32_t a_hi, uint32_t a_lo, uint64_t b_hi, uint64_t b_lo,
+                                        uint32_t idesc, uint32_t acc0) {
+#pragma unroll
+  for (int k = 0; k < KH; ++k) mma_ts_warp_tf32(d, a_hi + 8u * k, b_hi + 16u * k, idesc, k > 0 ? 1u : acc0);
+#pragma unroll
+  for (int k = 0; k < KX; ++k) mma_ts_warp_tf32(d, a_hi + 8u * k, b_lo + 16u * k, idesc, 1u);
+#pragma unroll
+  for (int k = 0; k < KX; ++k) mma_ts_warp_tf32(d, a_lo + 8u * k, b_hi + 16u * k, idesc, 1u);
+}
+
 // `steps` MMAs of K = 16 along one K extent; S > 0 unrolls a compile-time count.
 template <int S>
 __device__ __forceinline__ void mma_steps(int steps, uint32_t d_tmem, uint32_t a_tmem, uint64_t desc,
@@ -330,6 +374,39 @@ __device__ __forceinline__ void hidden_epilogue(int width, uint32_t src, uint32_
   }
 }
 
+// The exact fp32 variant's hidden epilogue: fp32 accumulators [0, W) at `src` -> ReLU
+// (NaN kept) -> tf32 hi part at `dst_hi`, the rest (fp32; the tensor core reads its top
+// tf32 bits) at `dst_lo`, one column per value.
+template <int W, class FL, class FS>
+__device__ __forceinline__ void hidden_epilogue_tf(uint32_t src, uint32_t dst_hi, uint32_t dst_lo, FL after_load,
+                                                   FS before_store) {
+  static_assert(W > 0 && W % 32 == 0, "32-column chunks");
+  uint32_t a[W / 32][32];
+#pragma unroll
+  for (int c = 0; c < W / 32; ++c) tmem_ld_x32(src + 32 * c, a[c]);
+  tmem_wait_ld();
+  after_load();
+  before_store();
+#pragma unroll
+  for (int c = 0; c < W / 32; ++c) {
+    uint32_t h[32], l[32];
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      const float v = __uint_as_float(a[c][j]);
+      const float r = v < 0.f ? 0.f : v;
+      h[j] = tf32_bits(r);
+      l[j] = __float_as_uint(r - __uint_as_float(h[j]));
+    }
+    tmem_st_x32(dst_hi + 32 * c, h);
+    tmem_st_x32(dst_lo + 32 * c, l);
+  }
+}
+
+// The aggregate words of a tile's A1 rows: h (and for the tf32 variant l, the lo parts).
+struct AggW {
+  uint4 h, l;
+};
+
 // KW: 32-bit words of an A1 row (8 or 16); AWO: word where the aggregate starts, or
 // -1 to take it from T at run time.  S1, S2, S3: K-steps of the three layers (0 = run time).
 // N3: columns of the layer-3 accumulator (16, or 0 = run time).  MP: the models run in
@@ -349,11 +426,14 @@ __device__ __forceinline__ void hidden_epilogue(int width, uint32_t src, uint32_
 // the previous tile's last, and that tile's constraints and top-k), a stage of the next
 // tile's digits and aggregate, and the next A1 row; then D2 -> H2.  The issuing warp does
 // nothing else, so an MMA group starts as soon as its operands are stored.
-template <int MODE, int KW, int AWO, int S1, int S2, int S3, int N3, bool MP, bool UT, int NM>
-__global__ void __launch_bounds__(kTcMaxPipes * kTcPipeThreads, 1)
+template <int MODE, int KW, int AWO, int S1, int S2, int S3, int N3, bool MP, bool UT, int NM, bool TF>
+__global__ void __launch_bounds__((TF ? 2 : kTcMaxPipes) * kTcPipeThreads, 1)
 k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   static_assert(AWO < 0 || AWO == 4 || AWO == 8, "partial A1 rows are written for these layouts only");
   static_assert(NM <= 7, "packed digits hold at most seven models");
+  static_assert(!TF || (KW == 16 && S1 == 2 && S2 == 9 && S3 == 8 && N3 == 16),
+                "the exact variant runs the d_L 8, 64-64 shape");
+  constexpr int KS = TF ? 8 : 16;  // K of one MMA
   // With the model count fixed at compile time (range mode), a tile's digits live in
   // registers, packed one per byte (model N - 1 in the lowest byte); otherwise in shared
   // memory, one byte per model and row, two tiles.
@@ -365,8 +445,8 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   __shared__ float s_b3[MF_MAX_MODELS][2];
   const int tid = threadIdx.x;
   // compile-time K-step counts must be the layout's (else no MMA may run)
-  if ((S1 > 0 && S1 != T.k1 / 16) || (S2 > 0 && S2 != T.h1 / 16 + 1) || (S3 > 0 && S3 != T.hl / 16) ||
-      (N3 > 0 && N3 != T.n3) || (NM > 0 && (NM != P.n_models || MP))) {
+  if ((S1 > 0 && S1 != T.k1 / KS) || (S2 > 0 && S2 != T.h1 / KS + 1) || (S3 > 0 && S3 != T.hl / KS) ||
+      (N3 > 0 && N3 != T.n3) || (NM > 0 && (NM != P.n_models || MP)) || TF != (T.tf != 0)) {
     if (tid == 0) atomicOr(P.status, kStatusBadInput);
     return;
   }
@@ -458,8 +538,10 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   const uint32_t tp = tmem + (uint32_t)(pipe * T.pipe_stride);
   const uint32_t lane_off = (uint32_t)(wq * 32) << 16;
   const uint32_t tD = tp + T.col_d, tA = tp + T.col_a, tD3 = tp + T.col_d3, tOnes = tp + T.col_ones;
-  const uint32_t tH1 = tOnes - (uint32_t)(T.h1 / 2);                        // layer-2 A operand
-  const uint32_t tH2 = T.h2 > 0 ? tOnes - (uint32_t)(T.h2 / 2) : tH1;       // layer-3 A operand
+  // layer-2 and layer-3 A operands (bf16 pairs, or tf32 hi parts with their lo parts at tHlo)
+  const uint32_t tH1 = tOnes - (uint32_t)(TF ? T.h1 : T.h1 / 2);
+  const uint32_t tH2 = T.h2 > 0 ? tOnes - (uint32_t)(TF ? T.h2 : T.h2 / 2) : tH1;
+  const uint32_t tHlo = tp + T.col_hlo;
   uint64_t* barA = &bars[1 + 2 * pipe];  // layers 1 and 2 completed (alternating)
   uint64_t* barB = &bars[2 + 2 * pipe];  // layer 3 completed
   uint32_t phA = 0, phB = 0;
@@ -470,13 +552,21 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   // and leave it waiting at the next one; the pipeline's top-k uses a third barrier
   // among its epilogue warps
   const int sig0 = 1 + 2 * pipe, barid = 1 + 2 * npipes + pipe;
-  const uint32_t id1 = idesc_bf16(T.h1), id2 = idesc_bf16(T.h2), id3 = idesc_bf16(T.n3);
-  const int s1 = T.k1 / 16, s2 = T.h1 / 16 + 1, s3 = T.hl / 16;
+  const uint32_t id1 = TF ? idesc_tf32(T.h1) : idesc_bf16(T.h1), id2 = TF ? idesc_tf32(T.h2) : idesc_bf16(T.h2),
+                 id3 = TF ? idesc_tf32(T.n3) : idesc_bf16(T.n3);
+  const int s1 = T.k1 / KS, s2 = T.h1 / KS + 1, s3 = T.hl / KS;
   const int m0 = MP ? T.m0 : 0, m1 = MP ? T.m1 : N;  // this pass's models
   const float vcap = P.vram_cap;
-  if (!issuer) {  // constant ones block: word 0 = (1, 1) feeds the bias hi/lo rows of B2
-    uint32_t v[8] = {0x3F803F80u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
-    tmem_st_x8(tOnes + lane_off, v);
+  if (!issuer) {  // constant ones block: (1, 1) feeds the bias hi/lo rows of B2
+    if constexpr (TF) {
+      uint32_t v[8] = {0x3F800000u, 0x3F800000u, 0u, 0u, 0u, 0u, 0u, 0u};
+      tmem_st_x8(tOnes + lane_off, v);
+      uint32_t z[32] = {};  // the A1 rows' unused words stay zero
+      tmem_st_x32(tA + lane_off, z);
+    } else {
+      uint32_t v[8] = {0x3F803F80u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
+      tmem_st_x8(tOnes + lane_off, v);
+    }
   }
   if (P.wait_test) mbar_wait_test(&bars[1 + 2 * npipes], P.wait_test, &s_abort, P.status);
 
@@ -491,17 +581,22 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   const uint32_t sb1 = smem_base;  // the pass's image starts with model m0's B1
   const uint32_t sb2 = smem_base + (T.off_b2[0] - T.off_b1[0]);
   const uint32_t sb3 = smem_base + (T.off_b3[0] - T.off_b1[0]);
+  // (tf32: 4 values per 16-byte core-matrix row, and each B image's lo part follows its hi part)
   auto issue_mma1 = [&](int i) {
-    mma_steps<S1>(s1, tD, tA, smem_desc(sb1 + (uint32_t)(i - m0) * T.img_model, 128u, (uint32_t)(T.k1 / 8) * 128u),
-                  id1, 0u);
+    const uint64_t b = smem_desc(sb1 + (uint32_t)(i - m0) * T.img_model, 128u, (uint32_t)(T.k1 / (TF ? 4 : 8)) * 128u);
+    if constexpr (TF) mma_tf3<S1, S1>(tD, tA, tA + 16u, b, b + (T.img_lo1 >> 4), id1, 0u);
+    else mma_steps<S1>(s1, tD, tA, b, id1, 0u);
   };
   auto issue_mma2 = [&](int i) {
-    mma_steps<S2>(s2, tD, tH1,
-                  smem_desc(sb2 + (uint32_t)(i - m0) * T.img_model, 128u, (uint32_t)((T.h1 + 16) / 8) * 128u), id2, 0u);
+    const uint64_t b = smem_desc(sb2 + (uint32_t)(i - m0) * T.img_model, 128u,
+                                 (uint32_t)((T.h1 + (TF ? 8 : 16)) / (TF ? 4 : 8)) * 128u);
+    if constexpr (TF) mma_tf3<S2, S2 - 1>(tD, tH1, tHlo, b, b + (T.img_lo2 >> 4), id2, 0u);
+    else mma_steps<S2>(s2, tD, tH1, b, id2, 0u);
   };
   auto issue_mma3 = [&](int i) {
-    mma_steps<S3>(s3, tD3, tH2, smem_desc(sb3 + (uint32_t)(i - m0) * T.img_model, 128u, (uint32_t)(T.hl / 8) * 128u),
-                  id3, i > m0 ? 1u : 0u);
+    const uint64_t b = smem_desc(sb3 + (uint32_t)(i - m0) * T.img_model, 128u, (uint32_t)(T.hl / (TF ? 4 : 8)) * 128u);
+    if constexpr (TF) mma_tf3<S3, S3>(tD3, tH2, tHlo, b, b + (T.img_lo3 >> 4), id3, i > m0 ? 1u : 0u);
+    else mma_steps<S3>(s3, tD3, tH2, b, id3, i > m0 ? 1u : 0u);
   };
   // The epilogue warps wait on the commits' mbarriers (suspended until the phase completes).
   auto await_a = [&]() {
@@ -540,8 +635,23 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     if constexpr (RD) return (uint32_t)(ds >> (8 * (NM - 1 - i))) & 0xFFu;
     else return ds[i * 128 + row];
   };
-  auto write_a1 = [&](int i, DS dg, bool with_agg, uint4 aw4) {
+  auto write_a1 = [&](int i, DS dg, bool with_agg, AggW aw) {
     const uint4* src = xw_s + (size_t)(P.off[i] + dig(dg, i)) * (KW >> 2);
+    if constexpr (TF) {  // words 0-7: x hi, 8-11: aggregate hi and 1; 16-23: x lo, 24-27: aggregate lo
+      const uint4 a = src[0], b = src[1], c = src[2], d = src[3];
+      const uint32_t vh[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+      const uint32_t vl[8] = {c.x, c.y, c.z, c.w, d.x, d.y, d.z, d.w};
+      tmem_st_x8(tA + lane_off, vh);
+      tmem_st_x8(tA + 16u + lane_off, vl);
+      if (with_agg) {
+        const uint32_t ah[4] = {aw.h.x, aw.h.y, aw.h.z, aw.h.w};
+        const uint32_t al[4] = {aw.l.x, aw.l.y, aw.l.z, aw.l.w};
+        tmem_st_x4(tA + 8u + lane_off, ah);
+        tmem_st_x4(tA + 24u + lane_off, al);
+      }
+      return;
+    }
+    const uint4 aw4 = aw.h;
     if (AWO >= 0 && !with_agg) {
       uint32_t v[AWO > 0 ? AWO : 1];
 #pragma unroll
@@ -616,7 +726,7 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   };
   // The aggregate state of a tile (fp32, model order) as the A1 words: bf16 hi/lo pairs;
   // its VRAM component (the same sum, unscaled) is the candidate's VRAM demand.
-  auto tile_agg = [&](DS dg, float& vram) -> uint4 {
+  auto tile_agg = [&](DS dg, float& vram) -> AggW {
     float A0 = 0.f, A1 = 0.f, A2 = 0.f;
 #pragma unroll (NM > 0 ? NM : 1)
     for (int i = 0; i < N; ++i) {
@@ -625,11 +735,18 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     }
     vram = A1;
     const float v0 = A0 * P.agg_scale[0], v1 = A1 * P.agg_scale[1], v2 = A2 * P.agg_scale[2];
+    if constexpr (TF) {  // tf32 hi parts and 1.0; the lo parts
+      const uint32_t h0 = tf32_bits(v0), h1 = tf32_bits(v1), h2 = tf32_bits(v2);
+      return AggW{make_uint4(h0, h1, h2, 0x3F800000u),
+                  make_uint4(__float_as_uint(v0 - __uint_as_float(h0)), __float_as_uint(v1 - __uint_as_float(h1)),
+                             __float_as_uint(v2 - __uint_as_float(h2)), 0u)};
+    }
     const uint32_t h0 = bf16_bits(v0), h1 = bf16_bits(v1), h2 = bf16_bits(v2);
     const uint32_t l0 = bf16_bits(v0 - __uint_as_float(h0 << 16));
     const uint32_t l1 = bf16_bits(v1 - __uint_as_float(h1 << 16));
     const uint32_t l2 = bf16_bits(v2 - __uint_as_float(h2 << 16));
-    return make_uint4(h0 | (h1 << 16), h2 | (0x3F80u << 16) /* bf16 1.0 */, l0 | (l1 << 16), l2);
+    return AggW{make_uint4(h0 | (h1 << 16), h2 | (0x3F80u << 16) /* bf16 1.0 */, l0 | (l1 << 16), l2),
+                make_uint4(0u, 0u, 0u, 0u)};
   };
   // Digits of a pipeline's first tile and its first A1 row (model m0) with the aggregate words.
   auto load_tile = [&](uint64_t tile, uint8_t* into, float& vram) -> DS {
@@ -639,8 +756,8 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   };
   // the model-i A1 row of the current tile (aggregate words already in place when AWO >= 0)
   auto next_a1 = [&](int i, DS dg) {
-    if (AWO >= 0) {
-      write_a1(i, dg, false, make_uint4(0u, 0u, 0u, 0u));
+    if (TF || AWO >= 0) {
+      write_a1(i, dg, false, AggW{});
     } else {  // run-time layout: the whole row, aggregate recomputed
       float A0 = 0.f, A1 = 0.f, A2 = 0.f;
       for (int j = 0; j < N; ++j) {
@@ -652,7 +769,7 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
       const uint32_t l0 = bf16_bits(v0 - __uint_as_float(h0 << 16));
       const uint32_t l1 = bf16_bits(v1 - __uint_as_float(h1 << 16));
       const uint32_t l2 = bf16_bits(v2 - __uint_as_float(h2 << 16));
-      write_a1(i, dg, true, make_uint4(h0 | (h1 << 16), h2 | (0x3F80u << 16), l0 | (l1 << 16), l2));
+      write_a1(i, dg, true, AggW{make_uint4(h0 | (h1 << 16), h2 | (0x3F80u << 16), l0 | (l1 << 16), l2), {}});
     }
   };
 
@@ -661,6 +778,7 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
   // landed, and its terms join this thread's running objective for the tile; later
   // models' layer-3 MMAs add zero to those columns.
   const int half3 = N3 == 16 ? 8 : (T.n3 >> 1);
+  constexpr float kBand = TF ? 0.f : 2e-2f;
   float acc_J = 0.f, acc_pen = 0.f;
   bool acc_ok = true, acc_near = true;
   // (the two loads are issued first; other work may run before `add_model` waits for them)
@@ -684,14 +802,14 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
       acc_J += util_term(P, j, P.off[j] + dig(dg, j), thr, &f);
       const float tau = P.u_tau[j];
       acc_ok = acc_ok && (f >= tau);
-      acc_near = acc_near && (f >= tau - 2e-2f * fmaxf(fabsf(tau), fabsf(f)));
+      acc_near = acc_near && (f >= tau - kBand * fmaxf(fabsf(tau), fabsf(f)));
       return;
     }
     acc_J = fmaf(P.w[j], thr, acc_J);
     const float sla = P.sla[j];
     acc_ok = acc_ok && (lat <= sla);
-    // shortlist test: within the bf16 error band of the ceiling
-    acc_near = acc_near && (lat <= sla + 2e-2f * fmaxf(fabsf(sla), fabsf(lat)));
+    // shortlist test: within the bf16 error band of the ceiling (none for the exact variant)
+    acc_near = acc_near && (lat <= sla + kBand * fmaxf(fabsf(sla), fabsf(lat)));
     const float over = lat - sla;
     acc_pen += over > 0.f ? over : 0.f;
   };
@@ -815,7 +933,7 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
     // while one model's layer 2 runs
     const int st_dig = m0 + 1 < m1 ? m0 + 1 : m1 - 1;
     const int st_agg = m0 + 2 < m1 ? m0 + 2 : m1 - 1;
-    uint4 aw_nx = make_uint4(0u, 0u, 0u, 0u);
+    AggW aw_nx{};
     for (; tile * 128 < n; tile += gstride) {
       uint8_t* buf_nx = digits + (buf ^ 1) * (MF_MAX_MODELS * 128);  // (shared-memory digits)
       const bool has_next = (tile + gstride) * 128 < n;
@@ -852,9 +970,15 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
         const bool next_l1 = i + 1 < m1 || has_next;
         // ---- layer 1 of model i landed: D1 -> H1 ----
         await_a();
-        hidden_epilogue<(S2 > 0 ? (S2 - 1) * 16 : 0)>(T.h1, tD + lane_off, tH1 + lane_off, []() {}, [&]() {
-          if (l3) await_b();  // the previous model's layer 3 has read H
-        });
+        if constexpr (TF) {
+          hidden_epilogue_tf<(S2 - 1) * 8>(tD + lane_off, tH1 + lane_off, tHlo + lane_off, []() {}, [&]() {
+            if (l3) await_b();  // the previous model's layer 3 has read H
+          });
+        } else {
+          hidden_epilogue<(S2 > 0 ? (S2 - 1) * 16 : 0)>(T.h1, tD + lane_off, tH1 + lane_off, []() {}, [&]() {
+            if (l3) await_b();  // the previous model's layer 3 has read H
+          });
+        }
         if (T.h2 == 0) {  // one hidden layer: the next layer 1, then layer 3 of model i
           side_work(i);
           if (next_l1) signal();
@@ -865,12 +989,21 @@ k_score_tc(const Params P, const TcArgs T, const RangeArgs R, const TcList L) {
         side_work(i);
         // ---- layer 2 of model i landed: D2 -> H2 ----
         await_a();
-        hidden_epilogue<(S3 > 0 ? S3 * 16 : 0)>(
-            T.h2, tD + lane_off, tH2 + lane_off,
-            [&]() {
-              if (next_l1) signal();  // accumulators read, next A1 written: the next layer 1
-            },
-            []() {});
+        if constexpr (TF) {
+          hidden_epilogue_tf<S3 * 8>(
+              tD + lane_off, tH2 + lane_off, tHlo + lane_off,
+              [&]() {
+                if (next_l1) signal();  // accumulators read, next A1 written: the next layer 1
+              },
+              []() {});
+        } else {
+          hidden_epilogue<(S3 > 0 ? S3 * 16 : 0)>(
+              T.h2, tD + lane_off, tH2 + lane_off,
+              [&]() {
+                if (next_l1) signal();  // accumulators read, next A1 written: the next layer 1
+              },
+              []() {});
+        }
         signal();  // H2 stored: layer 3 of model i
       }
       pending = true;
@@ -947,6 +1080,23 @@ size_t umma_off(int r, int k, int kdim) {
          (size_t)(k & 7) * 2u;
 }
 
+// The same for 4-byte (tf32) elements: 4 per 16-byte core-matrix row.
+size_t umma_off4(int r, int k, int kdim) {
+  return (size_t)(r >> 3) * (size_t)(kdim / 4) * 128u + (size_t)(k >> 2) * 128u + (size_t)(r & 7) * 16u +
+         (size_t)(k & 3) * 4u;
+}
+
+// v rounded to tf32 (nearest, ties away from zero), as an fp32 value.
+float tf32_round(double v) {
+  const float f = (float)v;
+  uint32_t u;
+  std::memcpy(&u, &f, 4);
+  if ((u & 0x7F800000u) != 0x7F800000u) u = (u + 0x1000u) & 0xFFFFE000u;  // (inf and NaN as they are)
+  float r;
+  std::memcpy(&r, &u, 4);
+  return r;
+}
+
 int round_up(int v, int a) { return (v + a - 1) / a * a; }
 
 size_t topk_bytes_pipe(int kcap, int qcap) {
@@ -980,7 +1130,7 @@ void layout_smem(const Params& P, TcArgs& T, int kcap) {
   T.kcap = kcap;
 }
 
-constexpr size_t kPassImageBudget = 160 * 1024;      // bf16 weights staged per pass
+constexpr size_t kPassImageBudget = 160 * 1024;      // weights staged per pass
 
 using TcFn = void (*)(const Params, const TcArgs, const RangeArgs, const TcList);
 
@@ -988,17 +1138,19 @@ using TcFn = void (*)(const Params, const TcArgs, const RangeArgs, const TcList)
 // models) with all counts fixed at compile time, and a run-time fallback per A1 row width.
 template <int MODE, bool MP, bool UT>
 TcFn tc_kernel_mode(const TcArgs& T, int n_models) {
+  // the exact fp32 variant (d_L 8, 64-64): S1 = k1 / 8, S2 = h1 / 8 + 1, S3 = hl / 8
+  if (T.tf) return k_score_tc<MODE, 16, 8, 2, 9, 8, 16, MP, UT, 0, true>;
   // S1 = k1 / 16, S2 = h1 / 16 + 1 (the b2 step), S3 = hl / 16
   if (T.kw == 8 && T.dle == 8 && T.h1 == 64 && T.h2 == 64 && T.n3 == 16) {
     if constexpr (MODE == kTcRange && !MP && !UT) {
-      if (n_models == 6) return k_score_tc<MODE, 8, 4, 1, 5, 4, 16, MP, UT, 6>;  // the 24^6 workload's shape
+      if (n_models == 6) return k_score_tc<MODE, 8, 4, 1, 5, 4, 16, MP, UT, 6, false>;  // the 24^6 workload's shape
     }
-    return k_score_tc<MODE, 8, 4, 1, 5, 4, 16, MP, UT, 0>;
+    return k_score_tc<MODE, 8, 4, 1, 5, 4, 16, MP, UT, 0, false>;
   }
   if (T.kw == 16 && T.dle == 16 && T.h1 == 128 && T.h2 == 128 && T.n3 == 16)
-    return k_score_tc<MODE, 16, 8, 2, 9, 8, 16, MP, UT, 0>;
-  if (T.kw == 8) return k_score_tc<MODE, 8, -1, 0, 0, 0, 0, MP, UT, 0>;
-  return k_score_tc<MODE, 16, -1, 0, 0, 0, 0, MP, UT, 0>;
+    return k_score_tc<MODE, 16, 8, 2, 9, 8, 16, MP, UT, 0, false>;
+  if (T.kw == 8) return k_score_tc<MODE, 8, -1, 0, 0, 0, 0, MP, UT, 0, false>;
+  return k_score_tc<MODE, 16, -1, 0, 0, 0, 0, MP, UT, 0, false>;
 }
 
 template <bool UT>
@@ -1067,12 +1219,151 @@ bool tc_supported(const Params& P, std::string* why) {
   return true;
 }
 
+bool tc_exact_supported(const Params& P) {
+  return P.d_local == 8 && P.h1 == 64 && P.h2 == 64 && P.n_models <= 8;
+}
+
+bool tc_fits(const mf_ctx* c, int kcap) {
+  TcArgs T = c->tc;
+  layout_smem(c->P, T, kcap);
+  return T.sm_total <= kSmemLimit;
+}
+
 int tc_grid(const mf_ctx* c) { return c->num_sms * c->tc.pipes; }
 
-mf_status tc_prepare(mf_ctx* c) {
+namespace {
+
+// The exact fp32 variant's layout and operand images (d_L 8, 12 -> 64 -> 64 -> 2): every
+// operand as a tf32 hi part and the rest (a lo part, also tf32), so that hi.hi + hi.lo +
+// lo.hi carries about 22 bits of each product.
+mf_status tc_prepare_exact(mf_ctx* c) {
+  const Params& P = c->P;
+  TcArgs& T = c->tc;
+  const int N = P.n_models, dl = P.d_local, h1 = P.h1, h2 = P.h2, hl = h2, din = P.d_in;
+  T.tf = 1;
+  T.dle = dl;
+  T.k1 = 16;   // [x (8) | aggregate (3) | 1 | 0 0 0 0]
+  T.kw = 16;   // words per option: x hi (8), x lo (8)
+  T.h1 = h1;
+  T.h2 = h2;
+  T.hl = hl;
+  T.n3 = 16;
+  // TMEM columns of a pipeline: D (64 fp32) | H hi (64) | ones (8) | H lo (64) | A1 hi (16), A1 lo (16) | D3 (16)
+  T.col_d = 0;
+  T.col_h = h1;
+  T.col_ones = 2 * h1;
+  T.col_hlo = T.col_ones + 8;
+  T.col_a = T.col_hlo + h1;
+  T.col_d3 = round_up(T.col_a + 32, 16);
+  T.pipe_stride = round_up(T.col_d3 + T.n3, 32);
+  T.pipes = 512 / T.pipe_stride;
+  if (T.pipes > 2) T.pipes = 2;
+  // per model: B1 [h1 x 16], B2 [h2 x (h1 + 8)] (its last K-step holds b2 hi, lo against
+  // the ones block), B3 [16 x hl], each as a hi image followed by a lo image
+  const int k2 = h1 + 8;
+  const size_t b1 = (size_t)h1 * T.k1 * 4, b2 = (size_t)h2 * k2 * 4, b3 = (size_t)T.n3 * hl * 4;
+  T.img_lo1 = (uint32_t)b1;
+  T.img_lo2 = (uint32_t)b2;
+  T.img_lo3 = (uint32_t)b3;
+  std::vector<float> w(P.per_model * N);
+  cudaError_t e = cudaMemcpy(w.data(), P.w32, sizeof(float) * w.size(), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "tc_prepare: read weights");
+  std::vector<unsigned char> img;
+  auto put = [&](size_t base, size_t lo_off, int r, int k, int kdim, double v) {
+    const float hi = tf32_round(v), lo = tf32_round(v - (double)hi);
+    std::memcpy(img.data() + base + umma_off4(r, k, kdim), &hi, 4);
+    std::memcpy(img.data() + base + lo_off + umma_off4(r, k, kdim), &lo, 4);
+  };
+  const double s3 = P.agg_scale[3];
+  for (int i = 0; i < N; ++i) {
+    const float* W1 = w.data() + (size_t)i * P.per_model;
+    const float* bb1 = W1 + (size_t)h1 * din;
+    const float* W2 = bb1 + h1;
+    const float* bb2 = W2 + (size_t)h2 * h1;
+    const float* W3 = bb2 + h2;
+    T.off_b1[i] = (uint32_t)img.size();
+    img.resize(img.size() + 2 * b1, 0);
+    for (int j = 0; j < h1; ++j) {
+      for (int k = 0; k < dl + 3; ++k) put(T.off_b1[i], b1, j, k, T.k1, W1[(size_t)j * din + k]);
+      // the constant-1 column: b1 plus the weight of the constant feature N * s_3
+      put(T.off_b1[i], b1, j, dl + 3, T.k1, (double)bb1[j] + (double)W1[(size_t)j * din + dl + 3] * s3 * N);
+    }
+    T.off_b2[i] = (uint32_t)img.size();
+    img.resize(img.size() + 2 * b2, 0);
+    for (int j = 0; j < h2; ++j) {
+      for (int k = 0; k < h1; ++k) put(T.off_b2[i], b2, j, k, k2, W2[(size_t)j * h1 + k]);
+      // b2 as two tf32 values (hi, then the rest) in the hi image, against the ones (1, 1)
+      const float bh = tf32_round(bb2[j]), bl = tf32_round((double)bb2[j] - (double)bh);
+      std::memcpy(img.data() + T.off_b2[i] + umma_off4(j, h1, k2), &bh, 4);
+      std::memcpy(img.data() + T.off_b2[i] + umma_off4(j, h1 + 1, k2), &bl, 4);
+    }
+    T.off_b3[i] = (uint32_t)img.size();
+    img.resize(img.size() + 2 * b3, 0);
+    T.img_model = (uint32_t)(2 * (b1 + b2 + b3));
+    for (int k = 0; k < hl; ++k) {
+      put(T.off_b3[i], b3, i, k, hl, W3[k]);
+      put(T.off_b3[i], b3, T.n3 / 2 + i, k, hl, W3[hl + k]);
+    }
+  }
+  img.resize(round_up((int)img.size(), 16), 0);
+  T.img_total = (uint32_t)img.size();
+  T.npasses = 0;
+  T.pass_m[0] = 0;
+  for (int i = 0; i < N;) {
+    int j = i + 1;
+    while (j < N && (size_t)((j + 1 < N ? T.off_b1[j + 1] : T.img_total) - T.off_b1[i]) <= kPassImageBudget) ++j;
+    T.pass_m[++T.npasses] = j;
+    i = j;
+  }
+  T.img_bytes = 0;
+  for (int p = 0; p < T.npasses; ++p) {
+    const uint32_t lo = T.off_b1[T.pass_m[p]];
+    const uint32_t hi = p + 1 < T.npasses ? T.off_b1[T.pass_m[p + 1]] : T.img_total;
+    if (hi - lo > T.img_bytes) T.img_bytes = hi - lo;
+  }
+  set_pass(T, 0, nullptr);
+  if (T.npasses == 1) { T.pass_last = 1; }
+  // option words: x hi (8), x lo (8)
+  const int sumK = c->sumK;
+  std::vector<float> x((size_t)sumK * dl);
+  e = cudaMemcpy(x.data(), P.x, sizeof(float) * x.size(), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "tc_prepare: read tables");
+  std::vector<float> xw((size_t)sumK * T.kw, 0.f);
+  for (int r = 0; r < sumK; ++r)
+    for (int k = 0; k < dl; ++k) {
+      const float v = x[(size_t)r * dl + k], hi = tf32_round(v);
+      xw[(size_t)r * T.kw + k] = hi;
+      xw[(size_t)r * T.kw + 8 + k] = tf32_round((double)v - (double)hi);
+    }
+  const size_t o_xw = round_up((int)img.size(), 256);
+  const size_t total = o_xw + round_up((int)(xw.size() * 4), 256);
+  MF_CUDA(cudaMalloc(&c->d_tc, total));
+  c->tc_bytes = total;
+  unsigned char* base = static_cast<unsigned char*>(c->d_tc);
+  MF_CUDA(cudaMemcpy(base, img.data(), img.size(), cudaMemcpyHostToDevice));
+  MF_CUDA(cudaMemcpy(base + o_xw, xw.data(), xw.size() * 4, cudaMemcpyHostToDevice));
+  c->stats.h2d_bytes_create += img.size() + xw.size() * 4;
+  T.img = base;
+  T.xw = reinterpret_cast<const uint32_t*>(base + o_xw);
+  for (int u = 0; u < 2; ++u) {
+    MF_CUDA(cudaFuncSetAttribute(tc_kernel(kTcRange, T, u, P.n_models), cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit));
+    MF_CUDA(cudaFuncSetAttribute(tc_kernel(kTcList, T, u, P.n_models), cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit));
+  }
+  layout_smem(P, T, 0);
+  if (T.sm_total > kSmemLimit) {
+    set_error("exact tensor-core path: tables and weights exceed shared memory");
+    return MF_EUNSUPPORTED;
+  }
+  return MF_OK;
+}
+
+}  // namespace
+
+mf_status tc_prepare(mf_ctx* c, bool exact) {
   const Params& P = c->P;
   TcArgs& T = c->tc;
   std::memset(&T, 0, sizeof(T));
+  if (exact) return tc_prepare_exact(c);
   const int N = P.n_models, dl = P.d_local, h1 = P.h1, h2 = P.h2, hl = h2 > 0 ? h2 : h1;
   const int din = P.d_in;
   T.dle = dl + (dl & 1);

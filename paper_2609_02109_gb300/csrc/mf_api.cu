@@ -121,7 +121,8 @@ mf_status mf_create(const mf_problem* p, mf_ctx** out) {
   if (p->objective != MF_OBJ_WEIGHTED_THR && p->objective != MF_OBJ_SOFT_LAT)
     return einval("unknown objective");
   if (p->out_act != MF_ACT_IDENTITY && p->out_act != MF_ACT_SIGMOID) return einval("unknown out_act");
-  if (p->precision != MF_FP32 && p->precision != MF_BF16) return einval("unknown precision");
+  if (p->precision != MF_FP32 && p->precision != MF_BF16 && p->precision != MF_FP32_SIMT)
+    return einval("unknown precision");
   if (std::isnan(p->vram_cap)) return einval("vram_cap is NaN");
   uint64_t total = 1;
   int sumK = 0;
@@ -245,6 +246,14 @@ mf_status mf_create(const mf_problem* p, mf_ctx** out) {
     } else {
       st3 = tc_prepare(c);
     }
+  } else if (st3 == MF_OK && c->precision == MF_FP32 && tc_exact_supported(P)) {
+    // the exact tensor-core variant where its operands fit; else the CUDA-core path
+    if (tc_prepare(c, true) != MF_OK) {
+      cudaFree(c->d_tc);
+      c->d_tc = nullptr;
+      std::memset(&c->tc, 0, sizeof(c->tc));
+      g_last_error.clear();
+    }
   }
   if (st3 != MF_OK) {
     free_ctx(c);
@@ -329,7 +338,7 @@ mf_status mf_score_batch(mf_ctx* ctx, const uint64_t* d_idx, uint64_t n, float* 
   if (!d_idx || !d_score) return einval("d_idx and d_score are required");
   DeviceGuard guard(ctx->device);
   cudaStream_t s = (cudaStream_t)stream;
-  if (ctx->precision == MF_BF16) return tc_score_list(ctx, d_idx, n, d_score, d_feasible, d_pred, s);
+  if (ctx->precision == MF_BF16 || ctx->tc.tf) return tc_score_list(ctx, d_idx, n, d_score, d_feasible, d_pred, s);
   float* pred = d_pred;
   const uint64_t tasks = n * (uint64_t)ctx->P.n_models;
   if (!pred && tasks <= 64ull * 1024) {
@@ -377,8 +386,10 @@ static mf_status search_impl(mf_ctx* ctx, uint64_t lo, uint64_t hi, int32_t k, u
   DeviceGuard guard(ctx->device);
   cudaStream_t s = (cudaStream_t)stream;
   const bool tc = !fc && ctx->precision == MF_BF16;
+  // the exact (3-term tf32) tensor-core variant, where its lists fit next to the weights
+  const bool tx = !fc && !tc && ctx->tc.tf && tc_fits(ctx, k);
   const int kcap = tc ? (k * 8 > 256 ? k * 8 : 256) : k;
-  const int grid = fc ? fc_grid(ctx) : tc ? tc_grid(ctx) : f32_grid(ctx);
+  const int grid = fc ? fc_grid(ctx) : (tc || tx) ? tc_grid(ctx) : f32_grid(ctx);
 
   // scratch: per-CTA lists, two merge buffers, merged list, rescored shortlist, count
   const size_t entries = (size_t)grid * kcap;
@@ -424,7 +435,7 @@ static mf_status search_impl(mf_ctx* ctx, uint64_t lo, uint64_t hi, int32_t k, u
     a.base = lo;
     a.len = 0;
     int nl = 1;
-    st = fc ? fc_search_chunk(ctx, a, s) : tc ? tc_search_chunk(ctx, a, s, &nl) : f32_search_chunk(ctx, a, s);
+    st = fc ? fc_search_chunk(ctx, a, s) : (tc || tx) ? tc_search_chunk(ctx, a, s, &nl) : f32_search_chunk(ctx, a, s);
     if (st != MF_OK) return st;
     launches += nl;
     score_launches += nl;
@@ -433,7 +444,7 @@ static mf_status search_impl(mf_ctx* ctx, uint64_t lo, uint64_t hi, int32_t k, u
     a.base = b;
     a.len = (hi - b) < chunk ? (hi - b) : chunk;
     int nl = 1;
-    st = fc ? fc_search_chunk(ctx, a, s) : tc ? tc_search_chunk(ctx, a, s, &nl) : f32_search_chunk(ctx, a, s);
+    st = fc ? fc_search_chunk(ctx, a, s) : (tc || tx) ? tc_search_chunk(ctx, a, s, &nl) : f32_search_chunk(ctx, a, s);
     if (st != MF_OK) return st;
     a.first = 0;
     launches += nl;
@@ -573,6 +584,7 @@ mf_status mf_ga_run(mf_ctx* ctx, const mf_ga_params* g, uint64_t seed, int32_t* 
 mf_status mf_get_stats(const mf_ctx* ctx, mf_stats* out) {
   if (!ctx || !out) return einval("NULL argument");
   *out = ctx->stats;
+  out->scoring_path = ctx->precision == MF_BF16 ? 1 : ctx->tc.tf ? 2 : 0;
   return MF_OK;
 }
 

@@ -46,12 +46,17 @@ struct Params {
 
 // Tensor-core path: operand images and the per-CTA layout (filled by tc_prepare).
 struct TcArgs {
-  const void* img;                    // bf16 B operands, UMMA K-major no-swizzle layout
+  const void* img;                    // B operands (bf16, or tf32 hi/lo), UMMA K-major no-swizzle layout
   uint32_t img_bytes;
-  const uint32_t* xw;                 // [sumK][kw] bf16 pairs of the local features
+  const uint32_t* xw;                 // [sumK][kw] local features: bf16 pairs, or tf32 hi then lo words
   int32_t k1, kw, h1, h2, hl, n3, dle;
   uint32_t off_b1[MF_MAX_MODELS], off_b2[MF_MAX_MODELS], off_b3[MF_MAX_MODELS];  // bytes in img
   int32_t pipes, col_d, col_h, col_ones, col_a, col_d3, pipe_stride;  // TMEM columns
+  // the exact fp32 variant (3-term tf32 split): operands as tf32 hi and lo parts; col_hlo
+  // holds the hidden layer's lo parts, img_lo1..3 are the byte offsets of each B image's
+  // lo part after its hi part
+  int32_t tf, col_hlo;
+  uint32_t img_lo1, img_lo2, img_lo3;
   uint32_t sm_xw, sm_dem, sm_rows, sm_topk, sm_bar, sm_total;  // shared-memory byte offsets
   uint32_t img_model;                 // bytes of one model's B1 + B2 + B3 images
   int32_t kcap;                       // per-pipeline list length the layout was sized for
@@ -444,7 +449,9 @@ mf_status select_topk(mf_ctx* c, const float* in_s, const uint64_t* in_i, int n,
 
 // Tensor-core scorer (bf16 path).
 bool tc_supported(const Params& P, std::string* why);
-mf_status tc_prepare(mf_ctx* c);
+bool tc_exact_supported(const Params& P);  // the exact fp32 (3-term tf32) variant's shapes
+bool tc_fits(const mf_ctx* c, int kcap);    // the context's tensor-core layout with lists of kcap
+mf_status tc_prepare(mf_ctx* c, bool exact = false);
 int tc_grid(const mf_ctx* c);
 mf_status tc_search_chunk(mf_ctx* c, const RangeArgs& a, cudaStream_t s, int* nlaunch);
 mf_status tc_score_list(mf_ctx* c, const uint64_t* idx, uint64_t n, float* score,

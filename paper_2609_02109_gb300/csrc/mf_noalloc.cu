@@ -90,7 +90,8 @@ extern "C" mf_status mf_search_exhaustive_noalloc(const mf_problem* p, int32_t k
   if (p->hidden2 < 0 || p->hidden2 > MF_MAX_HIDDEN) return einval("hidden2 must be in 0..256");
   if (p->objective != MF_OBJ_WEIGHTED_THR && p->objective != MF_OBJ_SOFT_LAT) return einval("unknown objective");
   if (p->out_act != MF_ACT_IDENTITY && p->out_act != MF_ACT_SIGMOID) return einval("unknown out_act");
-  if (p->precision != MF_FP32) return einval("the no-allocation search runs the fp32 path only");
+  if (p->precision != MF_FP32 && p->precision != MF_FP32_SIMT)
+    return einval("the no-allocation search runs the fp32 path only");
   if (p->vram_cap != p->vram_cap) return einval("vram_cap is NaN");
   if (k < 1 || k > MF_NOALLOC_MAX_TOPK) return einval("k must be in 1..64 for the no-allocation search");
 

@@ -18,7 +18,8 @@ from . import build as _build
 LIB_PATH = _build.LIB_PATH
 
 MF_OK, MF_EINVAL, MF_ENOMEM, MF_ECUDA, MF_EUNSUPPORTED, MF_ETIMEOUT, MF_EDEVICE = range(7)
-MF_FP32, MF_BF16 = 0, 1
+MF_FP32, MF_BF16, MF_FP32_SIMT = 0, 1, 2
+_PRECISIONS = {"fp32": MF_FP32, "bf16": MF_BF16, "fp32_simt": MF_FP32_SIMT}
 EMPTY = (1 << 64) - 1
 
 _EXPORTS = ["mf_status_string", "mf_last_error", "mf_create", "mf_destroy", "mf_space_size",
@@ -54,7 +55,7 @@ class _Result(C.Structure):
 class _Stats(C.Structure):
     _fields_ = [("h2d_bytes_create", C.c_uint64), ("d2h_bytes_last", C.c_uint64),
                 ("kernel_launches_last", C.c_int32), ("score_launches_last", C.c_int32),
-                ("score_ms_last", C.c_float), ("total_ms_last", C.c_float)]
+                ("score_ms_last", C.c_float), ("total_ms_last", C.c_float), ("scoring_path", C.c_int32)]
 
 
 class _GAParams(C.Structure):
@@ -150,7 +151,7 @@ def _problem_struct(prob: dict, device: int, prec: str):
                  float(prob["vram_cap"]), float(prob.get("soft_penalty", 0.0)),
                  1 if prob.get("out_act", "identity") == "sigmoid" else 0,
                  1 if prob.get("objective", "weighted_thr") == "soft_lat" else 0,
-                 MF_BF16 if prec == "bf16" else MF_FP32, int(device))
+                 _PRECISIONS[prec], int(device))
     return p, keep
 
 

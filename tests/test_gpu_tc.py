@@ -119,9 +119,11 @@ def test_tc_chunk_invariance(mf, chunk):
 
 def test_tc_and_fp32_paths_agree_on_large_range(mf):
     """A 2^22-candidate range of the N=6 workload searched by both paths: the
-    re-scored bf16 top-k equals the fp32 top-k."""
+    re-scored bf16 top-k equals the fp32 top-k (the bf16 path re-scores its shortlist
+    with the CUDA-core fp32 kernels, so against precision fp32_simt)."""
     lo, hi = 24 ** 6 // 2, 24 ** 6 // 2 + (1 << 22)
-    with mf.Context(W.large(precision="fp32")) as c32, mf.Context(W.large(precision="bf16")) as c16:
+    with mf.Context(W.large(precision="fp32"), precision="fp32_simt") as c32, \
+            mf.Context(W.large(precision="bf16")) as c16:
         a = c32.search(32, lo=lo, hi=hi)
         b = c16.search(32, lo=lo, hi=hi)
     assert a["count"] == b["count"] == hi - lo

@@ -4,7 +4,8 @@ holds the GPU's memory, or a control loop that must not pay cudaMalloc's implici
 synchronisation).  It keeps all of its device memory in one fixed array inside the
 library.  Its results must equal those of the regular entry point,
 mf_search_exhaustive, on every call, including consecutive calls that reuse the
-array left behind by the previous one.
+array left behind by the previous one.  It runs the CUDA-core fp32 kernels, so it is
+compared with contexts of precision "fp32_simt".
 
 This file is named to be collected last, so a run that stops at the first failure
 has already run every other test."""
@@ -47,8 +48,8 @@ def _same(got, ref):
 def test_noalloc_equals_regular_search_on_consecutive_calls(mf, k):
     problems = [W.tiny(), _tight(), W.paper_scale()]
     refs = []
-    for prob in problems:
-        with mf.Context(prob) as ctx:
+    for prob in problems:  # (the same CUDA-core fp32 kernels)
+        with mf.Context(prob, precision="fp32_simt") as ctx:
             refs.append(ctx.search(k))
     # two calls in a row on each problem, then the problems in a different order:
     # each call must clear what the previous call left in the shared array
