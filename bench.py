@@ -46,8 +46,10 @@ L2_FLUSH_BYTES = 256 << 20
 
 # DRAM bytes (read + write) of one scoring launch from the ncu capture of the scoring
 # kernel on this workload, valid only while the kernel's sources are the ones that were
-# captured (sha256 prefix of k_tc.cu + mf_internal.cuh)
-NCU_TRAFFIC = {"bf16": ("739c026bcbb59df6", 2116864)}
+# captured (sha256 prefix of k_tc.cu + mf_internal.cuh).  fp32: a first-pass launch of
+# the exact variant (models 0-2), which writes the 16-byte partial record of each of its
+# 2^24 candidates for the second pass (which reads them back).
+NCU_TRAFFIC = {"bf16": ("3ee8331533f0ffec", 2059008), "fp32": ("3ee8331533f0ffec", 208286208)}
 
 
 def _traffic(prec):
@@ -278,29 +280,58 @@ def tight_throughput(mf, torch, device):
                          "peak_source": f"{src} bf16 burst"}}
 
 
+# tf32 dense tensor rate relative to bf16 (NVIDIA's nominal 1.1 vs 2.25 PFLOP/s)
+TF32_PER_BF16 = 1.1 / 2.25
+
+
+def exact_roofline(achieved, sgemm_tflops):
+    """Roofline of the exact fp32 tensor-core variant: every product costs three tf32
+    products (hi.hi, hi.lo, lo.hi), so its ceiling is a third of the tf32 peak (the
+    measured bf16 burst x the nominal tf32 / bf16 ratio)."""
+    peaks, src = _peaks()
+    tf32 = float(peaks["bf16_tflops"]) * TF32_PER_BF16
+    return {"bound": "tensor", "achieved": achieved, "peak": tf32, "unit": "TFLOP/s", "frac": achieved / tf32,
+            "frac_of_split_ceiling": 3 * achieved / tf32,
+            "peak_source": f"{src} bf16 burst x {TF32_PER_BF16:.3f} (nominal tf32 / bf16); 3 tf32 products per product",
+            "cuda_core_peak": sgemm_tflops}
+
+
 def exact_throughput(mf, torch, device, sgemm_tflops):
-    """The exact fp32 search (CUDA-core scorer) of the large workload."""
+    """The exact fp32 search of the large workload: the tensor-core variant (3-term
+    tf32 split) and, for comparison, the CUDA-core scorer."""
     prob = W.large(precision="fp32")
     n = 24 ** 6
     stream = torch.cuda.current_stream(device)
-    with mf.Context(prob, device=device) as ctx:
-        ctx.search(K_TOP, chunk=CHUNK)
-        e0 = torch.cuda.Event(enable_timing=True)
-        e1 = torch.cuda.Event(enable_timing=True)
-        torch.cuda.synchronize(device)
-        e0.record(stream)
-        res = ctx.search(K_TOP, chunk=CHUNK)
-        e1.record(stream)
-        e1.synchronize()
-        st = ctx.stats()
-    ms = e0.elapsed_time(e1)
-    launch_ms = st["score_ms_last"] / st["score_launches_last"]
-    achieved = flops_per_candidate(prob) * (n / st["score_launches_last"]) / (launch_ms / 1e3) / 1e12
-    return {"workload": "large exhaustive, exact fp32 path", "value": n / (ms / 1e3), "unit": UNIT, "ms": ms,
-            "best": res["best_idx"], "count": res["count"],
-            "roofline": {"bound": "fp32", "achieved": achieved, "peak": sgemm_tflops, "unit": "TFLOP/s",
-                         "frac": achieved / sgemm_tflops, "launch_ms": launch_ms,
-                         "peak_source": "measured cuBLAS fp32 GEMM (TF32 off), this run"}}
+    out = {}
+    for prec in ("fp32", "fp32_simt"):
+        with mf.Context(prob, device=device, precision=prec) as ctx:
+            ctx.search(K_TOP, chunk=CHUNK)
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            torch.cuda.synchronize(device)
+            e0.record(stream)
+            res = ctx.search(K_TOP, chunk=CHUNK)
+            e1.record(stream)
+            e1.synchronize()
+            st = ctx.stats()
+        ms = e0.elapsed_time(e1)
+        launch_ms = st["score_ms_last"] / st["score_launches_last"]
+        achieved = flops_per_candidate(prob) * (n / st["score_launches_last"]) / (launch_ms / 1e3) / 1e12
+        out[prec] = dict(value=n / (ms / 1e3), ms=ms, best=res["best_idx"], count=res["count"],
+                         path=int(st["scoring_path"]), achieved=achieved, launch_ms=launch_ms,
+                         launches=int(st["score_launches_last"]))
+    tc, simt = out["fp32"], out["fp32_simt"]
+    roof = exact_roofline(tc["achieved"], sgemm_tflops) if tc["path"] == 2 else \
+        {"bound": "fp32", "achieved": tc["achieved"], "peak": sgemm_tflops, "unit": "TFLOP/s",
+         "frac": tc["achieved"] / sgemm_tflops, "peak_source": "measured cuBLAS fp32 GEMM (TF32 off), this run"}
+    roof["launch_ms"] = tc["launch_ms"]
+    return {"workload": "large exhaustive, exact fp32 path (tensor cores, 3-term tf32 split; "
+                        "two weight passes of three models)", "value": tc["value"], "unit": UNIT, "ms": tc["ms"],
+            "best": tc["best"], "count": tc["count"], "roofline": roof,
+            "cuda_cores": {"value": simt["value"], "unit": UNIT, "ms": simt["ms"], "best": simt["best"],
+                           "count": simt["count"], "achieved": simt["achieved"], "unit_achieved": "TFLOP/s",
+                           "frac": simt["achieved"] / sgemm_tflops,
+                           "peak_source": "measured cuBLAS fp32 GEMM (TF32 off), this run"}}
 
 
 def stress_throughput(mf, torch, device):
@@ -502,6 +533,7 @@ def run_gpu(args):
                 score_ms.append(st["score_ms_last"])
                 launches += st["kernel_launches_last"]
                 score_launches += st["score_launches_last"]
+            ctx_path = int(st["scoring_path"])
             torch.cuda.synchronize(device)
             if dist:
                 dist.barrier()
@@ -527,6 +559,8 @@ def run_gpu(args):
             roof = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                     "frac": achieved / peak, "frac_sustained": achieved / float(peaks["bf16_tflops_sustained"]),
                     "peak_source": f"{src} bf16 burst (sustained {peaks['bf16_tflops_sustained']})"}
+        elif ctx_path == 2:  # the exact tensor-core variant
+            roof = exact_roofline(achieved, sgemm)
         else:
             roof = {"bound": "fp32", "achieved": achieved, "peak": sgemm, "unit": "TFLOP/s",
                     "frac": achieved / sgemm if sgemm else None,
