@@ -1,4 +1,4 @@
-// Tensor-core (tcgen05, bf16 x bf16 -> fp32) scorer for sm_103a.
+// Tensor-core (tcgen05: bf16 x bf16 -> fp32, or 3-term tf32 -> fp32) scorer for sm_103a.
 //
 // Same computation as the exact fp32 path (arXiv 2609.02109: Eq. 1 decode, the
 // aggregate GPU state, the per-model MeanField MLP of Eq. 6, the constraints of
@@ -11,27 +11,36 @@
 //                                                    so D3 accumulates all N models
 //                                                    (b3 is added in the final epilogue).
 //
-// One persistent CTA per SM runs up to four independent 128-row pipelines of
-// four warps each (warp q of a pipeline owns TMEM lanes 32q..32q+31).  Each
-// pipeline keeps every A operand in tensor memory (layer inputs written with
-// tcgen05.st, hidden activations converted in place from the fp32 accumulators
-// with cvt.rn.relu.bf16x2), so the tensor core reads only the weights (B) from
-// shared memory.  The weights are staged once per CTA with one TMA bulk copy.
-// The pipeline's first thread issues the MMAs and commits them to an mbarrier
-// that the pipeline's threads wait on (bounded; a wait that gives up raises the
-// status word and the kernel runs to completion without further waits).
+// One persistent CTA per SM runs up to four independent 128-row pipelines.  Each has
+// four epilogue warps (warp q of a pipeline owns TMEM lanes 32q..32q+31) and one warp
+// that only issues the pipeline's MMAs: every MMA group starts on a named-barrier
+// rendezvous with the epilogue warps once its operands are stored, and is committed to
+// an mbarrier the epilogue warps wait on (bounded; a wait that gives up raises the
+// status word and the kernel runs to completion without further waits).  Every A
+// operand stays in tensor memory (layer inputs written with tcgen05.st, hidden
+// activations converted from the fp32 accumulators with cvt.rn.relu.bf16x2), so the
+// tensor core reads only the weights (B) from shared memory, staged once per CTA (per
+// pass of models) with TMA bulk copies.
 //
 // b1 rides in A1's constant-1 column and b2 in a constant block of ones that sits
 // in tensor memory right after H1 (one extra K = 16 step whose B rows hold the bias
 // as a bf16 hi/lo pair), so the hidden epilogues are only load -> ReLU + round ->
 // store.  b3 is added in fp32 in the final epilogue: a bias step of layer 3 would
-// cost a whole MMA issue (~60 cycles of the issuing thread) for two numbers.  The
-// aggregate enters layer 1 as a bf16 hi/lo pair as well (two columns per
-// component with the same weight), so its rounding error is ~2^-16, not 2^-9.
+// cost a whole MMA issue for two numbers.  The aggregate enters layer 1 as a bf16
+// hi/lo pair as well (two columns per component with the same weight), so its
+// rounding error is ~2^-16, not 2^-9.
 //
-// Each thread keeps its candidate's option rows in shared memory and steps them
+// Each thread keeps its candidate's digits (option index per model) and steps them
 // from tile to tile by adding the digits of the tile stride with carries, so no
-// division runs in the hot loop.
+// division runs in the hot loop: packed in registers in the six-model instantiation,
+// else in shared memory.
+//
+// The exact fp32 variant (TF) runs the same kernel on tf32 operands: every operand is
+// a tf32 hi part plus a tf32 lo part (the rest), and each K = 8 step issues
+// hi.hi + hi.lo + lo.hi MMAs of kind::tf32 into the fp32 accumulator (lo.lo, about
+// 2^-22 of a product, is dropped), which keeps the scores within the fp32 path's
+// 1e-5.  Its tensor-memory layout (256 columns per pipeline) leaves room for two
+// pipelines.
 #include <cuda_bf16.h>
 
 #include <cstring>
