@@ -532,6 +532,31 @@ k_fc_ga(const Params P, const FcGaArgs A) {
   const int c = threadIdx.x;
   for (int e = c; e < sumK; e += blockDim.x) tab[e] = A.tab[e];
   __syncthreads();
+  // Does any configuration meet the floors and the VRAM bound?  Exactly when every model
+  // has an option with a finite term and the smallest such VRAM demands, summed in model
+  // order as the fitness sums them, fit the cap (fp32 rounding is monotone, so no other
+  // configuration sums to less).  If none does, every repair would draw all its attempts
+  // in vain; its draws come from their own stream, so skipping it changes nothing else.
+  __shared__ int s_any_feasible;
+  if (c < 32) {
+    float V = 0.f;
+    bool every = true;
+    for (int i = 0; i < N; ++i) {
+      const int off = pick(P.off, i), K = pick(P.K, i);
+      float m = INFINITY;
+      for (int o = c; o < K; o += 32) {
+        const float2 e = tab[off + o];
+        if (e.x > -INFINITY && e.y < m) m = e.y;
+      }
+#pragma unroll
+      for (int w = 16; w > 0; w >>= 1) m = fminf(m, __shfl_xor_sync(0xffffffffu, m, w));
+      every = every && m < INFINITY;
+      V += m;
+    }
+    if (c == 0) s_any_feasible = every && V <= P.vram_cap ? 1 : 0;
+  }
+  __syncthreads();
+  const bool repairable = A.repair && s_any_feasible;
   const uint64_t sd = A.seed;
   const int attempts = 256 / N;
   // Repair of the generation's infeasible children (need): the cnt of them, in ascending
@@ -600,7 +625,7 @@ k_fc_ga(const Params P, const FcGaArgs A) {
     for (int i = 0; i < N; ++i) g[i] = (uint8_t)ga_unif(ga_rng(sd, 0, (uint32_t)c, kGaInit, (uint32_t)i), (uint32_t)pick(P.K, i));
     const float J = fc_fit(P, tab, g);
     fit0[c] = J;
-    need = A.repair && J == -INFINITY;
+    need = repairable && J == -INFINITY;
   }
   repair(0u, need, g0, fit0);
   __syncthreads();
@@ -642,7 +667,7 @@ k_fc_ga(const Params P, const FcGaArgs A) {
       }
       const float J = fc_fit(P, tab, g);
       fn[c] = J;
-      need = A.repair && J == -INFINITY;
+      need = repairable && J == -INFINITY;
     }
     repair(G, need, gn, fn);
     __syncthreads();

@@ -239,6 +239,38 @@ def test_paper_ga_reproduces_the_oracle_exactly(mf, oracle_mod, opts, params):
             assert list(g) == list(go) and J == Jo, (seed, g, go, J, Jo)
 
 
+@pytest.mark.parametrize("case", ["floor_unmet", "vram_short", "vram_exact"])
+def test_paper_ga_with_no_or_one_tier_of_feasible_configurations(mf, oracle_mod, case):
+    """The GA kernel skips repairs when no configuration can be feasible (its repair draws
+    have their own stream, so the run is the same as drawing every attempt in vain).
+    floor_unmet: model 0 has no option at its floor; vram_short: every floor can be met
+    but the smallest VRAM demands exceed the cap by 1; vram_exact: they equal the cap
+    (feasible, the bound being inclusive).  Each run equals the oracle's bit for bit."""
+    opts = [12, 9, 9, 9, 9]
+    prob = W.integer_landscape(opts, 5, 5.0 * len(opts) + 5.0)
+    fc = _integer_fc(prob, 7)
+    if case == "floor_unmet":
+        tau = np.asarray(fc["tau"], np.float32).copy()
+        tau[0] = 1e6
+        fc = dict(fc, tau=tau)
+    else:
+        _, _, rok, _ = oracle_mod.Oracle(prob).fc_local(fc)
+        off = np.concatenate([[0], np.cumsum(prob["n_options"])])
+        vram = np.asarray(prob["demand"], np.float64)[:, 1]
+        need = sum(float(vram[off[i]:off[i + 1]][rok[off[i]:off[i + 1]]].min()) for i in range(len(opts)))
+        prob = dict(prob, vram_cap=np.float32(need - 1.0 if case == "vram_short" else need))
+    o = oracle_mod.Oracle(prob)
+    _, _, cnt = o.fc_exhaustive(fc, 1)
+    assert (cnt == 0) == (case != "vram_exact")
+    params = dict(W.PAPER_GA_PARAMS, gens=12)
+    with mf.Context(prob) as ctx:
+        ctx.fc_set(fc)
+        for seed in (1000, 2 ** 40 + 9):
+            J, g = ctx.fc_ga_run(params, seed)
+            Jo, go = o.fc_ga_run(fc, params, seed)
+            assert list(g) == list(go) and (J == Jo or (np.isinf(J) and np.isinf(Jo))), (seed, g, go, J, Jo)
+
+
 def test_paper_ga_decisions_on_the_paper_landscape(mf, oracle_mod):
     """The synthetic N = 5 landscape: every decision's oracle score equals its reported
     fitness and is within 0.5 % of the exhaustive optimum."""
