@@ -68,12 +68,24 @@ def _create(mf, prob, **over):
     dict(n_models=0), dict(n_models=17), dict(n_options=np.array([12, 0], np.int32)),
     dict(n_options=np.array([12, 256], np.int32)), dict(d_local=0), dict(d_local=29),
     dict(hidden1=0), dict(hidden1=257), dict(hidden2=-1), dict(objective=2), dict(out_act=3),
-    dict(precision=7), dict(weights=None), dict(sla=None), dict(vram_cap=float("nan")),
+    dict(precision=7), dict(precision=3), dict(precision=-1), dict(weights=None), dict(sla=None),
+    dict(vram_cap=float("nan")),
 ])
 def test_create_rejects_bad_problems(mf, over):
     st, h = _create(mf, W.tiny(), **over)
     assert st == mf.MF_EINVAL and not h.value
     assert mf.lib().mf_last_error()
+
+
+@pytest.mark.parametrize("precision", [0, 1, 2])  # MF_FP32, MF_BF16, MF_FP32_SIMT
+def test_create_accepts_every_precision(mf, precision):
+    """Validation passes for the three precisions (without a device the call then fails
+    in the CUDA runtime, not in validation)."""
+    st, h = _create(mf, W.paper_scale(), precision=precision)
+    assert st != mf.MF_EINVAL, mf.lib().mf_last_error()
+    if st == mf.MF_OK:
+        mf.lib().mf_destroy(h)
+    assert mf.MF_FP32_SIMT == 2 and mf._PRECISIONS["fp32_simt"] == mf.MF_FP32_SIMT
 
 
 def test_create_rejects_space_overflow(mf):
