@@ -403,7 +403,9 @@ __device__ __forceinline__ void hidden_epilogue_tf(uint32_t src, uint32_t dst_hi
     for (int j = 0; j < 32; ++j) {
       const float v = __uint_as_float(a[c][j]);
       const float r = v < 0.f ? 0.f : v;
-      h[j] = tf32_bits(r);
+      // tf32 rounding, nearest with ties away from zero: half a tf32 ulp (2^12 in the
+      // fp32 bits) added to the magnitude, the 13 dropped bits cleared (r >= 0 or NaN)
+      h[j] = (__float_as_uint(r) + 0x1000u) & 0xFFFFE000u;
       l[j] = __float_as_uint(r - __uint_as_float(h[j]));
     }
     tmem_st_x32(dst_hi + 32 * c, h);
