@@ -257,8 +257,20 @@ __device__ __noinline__ void mbar_wait_slow(uint64_t* bar, uint32_t parity, vola
 struct PipeWait {
   volatile int* abort;
   uint32_t* status;
-  // Bounded wait for `parity` of `bar` (the usual case is one suspended try).
+  // Bounded wait for `parity` of `bar`: first up to 48 non-blocking polls (an MMA group
+  // usually completes within a few hundred cycles of the wait, and a polling warp sees
+  // it sooner than a suspended one is woken), then suspended tries.
   __device__ __forceinline__ void operator()(uint64_t* bar, uint32_t parity) const {
+    for (int i = 0; i < 48; ++i) {
+      uint32_t ok;
+      asm volatile(
+          "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+          " selp.u32 %0, 1, 0, p;\n}"
+          : "=r"(ok)
+          : "r"(smem_u32(bar)), "r"(parity)
+          : "memory");
+      if (ok) return;
+    }
     if (!mbar_try_wait(bar, parity)) mbar_wait_slow(bar, parity, abort, status);
   }
 };
