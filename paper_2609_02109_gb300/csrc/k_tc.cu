@@ -257,11 +257,11 @@ __device__ __noinline__ void mbar_wait_slow(uint64_t* bar, uint32_t parity, vola
 struct PipeWait {
   volatile int* abort;
   uint32_t* status;
-  // Bounded wait for `parity` of `bar`: first up to 48 non-blocking polls (an MMA group
+  // Bounded wait for `parity` of `bar`: first up to 96 non-blocking polls (an MMA group
   // usually completes within a few hundred cycles of the wait, and a polling warp sees
   // it sooner than a suspended one is woken), then suspended tries.
   __device__ __forceinline__ void operator()(uint64_t* bar, uint32_t parity) const {
-    for (int i = 0; i < 48; ++i) {
+    for (int i = 0; i < 96; ++i) {
       uint32_t ok;
       asm volatile(
           "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n"
